@@ -283,6 +283,12 @@ def test_pow2_is_nearest_power_and_bounds():
     x64, q64 = x.astype(np.float64), dec.astype(np.float64)
     assert np.linalg.norm(x64 - q64) <= 0.5 * np.linalg.norm(x64) + 2.0 ** k * np.sqrt(d)
     assert q.message_bits(d) == d * 4
+    # exact midpoints 1.5 * 2^j between two levels go up; just below them go down
+    mid = np.array([1.5 * 2.0 ** j for j in range(k, K)], np.float32)
+    qm = O.Quantizer(O.Q_POW2, bits, O.group_offsets(len(mid), 0), pow2_k=k, pow2_K=K)
+    np.testing.assert_array_equal(qm.quantize(mid)[2], (2 * mid / 1.5).astype(np.float32))
+    below = np.nextafter(mid, np.float32(0))
+    np.testing.assert_array_equal(qm.quantize(-below)[2], (-mid / 1.5).astype(np.float32))
     # The appendix bounds each coordinate's error by |x_j|/2, hence |Q(x)_j| <= 1.5 |x_j|, for
     # 2^(k-1) <= |x_j| <= 2^K + 2^(K-1).  Both hold from (2/3) 2^k upwards ...
     lo, hi = 2.0 ** k * 2.0 / 3.0, 2.0 ** K + 2.0 ** (K - 1)

@@ -131,7 +131,9 @@ def test_virtual_iterates_notation1():
         steps, decs = [], []
         for i in range(n):
             orc.worker_compress(i, gs[i])
-            steps.append(orc.last_input(i).astype(np.float64) - e_old[i])  # alpha m / sqrt(v)
+            # the Adam step alpha m / sqrt(v), from the moments (pinned by the closed-form test)
+            m, v = orc.m[i].astype(np.float64), orc.v[i].astype(np.float64)
+            steps.append(_f(1e-3) * m / np.sqrt(v))
             decs.append(orc.worker_decoded(i).astype(np.float64))
         orc.server_step()
         orc.apply(x)
