@@ -1,0 +1,456 @@
+"""Benchmark: rounds of Efficient-Adam's two-way quantized error-feedback pipeline on one GB300.
+
+One step = one full round: n worker compresses (Algorithm 2), the server step (Algorithm 1) and
+x <- x - Q_s(w), on the default workload c5 (d = 1,558,000,000 fp32 parameters, n = 8 workers,
+1-bit scaled sign with 4096-block scales, Adam moments on the workers).  The metric is round
+throughput in parameter x worker elements per second.  Inputs are synthetic and resident in HBM
+(the working set, ~213 GB, is far larger than the 129 MB L2, so no flush is needed between steps).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5] [--placement worker|server]
+    python bench.py --impl reference     # the oracle on the host cores, same metric
+
+With torchrun (N > 1) every rank runs an independent replica of the workload on its own GPU (the
+simulated round does not shard: replicas only); the value is the sum of elements over all ranks
+divided by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "round throughput (param x worker elems/s) and achieved HBM GB/s vs GB300 peak"
+UNIT = "param*worker elems/s"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _workload(name: str):
+    from paper_2205_14473_gb300 import workloads as W
+
+    return W.WORKLOADS[name]
+
+
+def _describe(w, placement: int) -> str:
+    from paper_2205_14473_gb300 import workloads as W
+
+    kinds = {W.Q_SIGN_L1: "1-bit scaled sign", W.Q_UNIFORM_MAX: "uniform grid", W.Q_POW2: "power-of-two",
+             W.Q_IDENTITY: "identity"}
+
+    def q(s):
+        g = "whole-vector" if s.group == 0 else (f"{s.group}-block" if s.group > 0 else "per-tensor")
+        extra = f" {s.bits}-bit{' stochastic' if s.stochastic else ''}" if s.kind == W.Q_UNIFORM_MAX else ""
+        return f"{kinds[s.kind]}{extra}, {g} scales"
+    where = "Adam at workers (Algorithm 2)" if placement == 0 else "Adam at server"
+    return f"{w.name}: d={w.d:,} fp32, n={w.n} workers; Q_w {q(w.qw)}; Q_s {q(w.qs)}; {where}"
+
+
+def algorithmic_bytes(w, placement: int) -> dict:
+    """Bytes per launch that each kernel must move at least (fp32 state, codes at b bits)."""
+    d, n = w.d, w.n
+    bw, bs = w.qw.bits / 8.0, w.qs.bits / 8.0
+    gw = 0 if w.qw.kind in (0, 3) else (1 if w.qw.group == 0 else (-(-d // w.qw.group) if w.qw.group > 0 else
+                                                                    len(w.qw.segments)))
+    gs = 0 if w.qs.kind in (0, 3) else (1 if w.qs.group == 0 else (-(-d // w.qs.group) if w.qs.group > 0 else
+                                                                    len(w.qs.segments)))
+    if placement == 0:
+        compress = d * (16 + 12 + bw) + 4 * gw      # g, m, v, e read; m, v, e written; codes + scales
+        server = d * (n * bw + 8 + bs) + 4 * (n * gw + gs)
+    else:
+        compress = d * (8 + 4 + bw) + 4 * gw        # g, e read; e written
+        server = d * (n * bw + 24 + bs) + 4 * (n * gw + gs)
+    apply = d * (8 + bs) + 4 * gs
+    return {"compress": compress, "server": server, "apply": apply,
+            "round": n * compress + server + apply}
+
+
+def _kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2205_14473_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def _ncu_traffic(kernel: str, workload: str, placement: int):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if it was taken on the
+    current kernel sources (profiles/ncu_traffic.txt: `kernel workload placement source-hash bytes`)."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    cur = _kernel_source_hash()
+    for line in open(path):
+        p = line.split()
+        if len(p) == 5 and not line.startswith("#") and p[0] == kernel and p[1] == workload and \
+                p[2] == str(placement) and p[3] == cur:
+            return float(p[4])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.samples = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            p = [x.strip() for x in line.split(",")]
+            if len(p) >= 9:
+                self.samples.append(p)
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(p[1]) for p in self.samples if p[1].replace(".", "").isdigit()]
+        mx = [float(p[2]) for p in self.samples if p[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for p in self.samples:
+            for name, v in zip(names, p[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(self.samples)}
+
+
+# ------------------------------------------------------------------------------- CPU baseline
+
+class OracleSample:
+    """The oracle, as it stands, on a bounded sample of the workload: `blocks` whole 4096-blocks of
+    every worker when the scales are per 4096-block (the round is separable by block; the global
+    coordinates key the Philox counters), else a prefix of d with the same quantizers.  One step()
+    is one full round (n worker steps, the server step, the update of x) on one host thread."""
+
+    def __init__(self, w, placement: int, blocks: int = 16):
+        import numpy as np
+
+        import oracle as O
+        from paper_2205_14473_gb300 import workloads as W
+
+        if w.qw.group == 4096 and w.qs.group == 4096:
+            sel = W.sample_blocks(w, blocks)
+            lens = np.array([min(4096, w.d - b * 4096) for b in sel], np.int64)
+            d = int(lens.sum())
+            offs = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+            gidx = np.concatenate([np.arange(b * 4096, b * 4096 + l) for b, l in zip(sel, lens)])
+            self.sample = f"{len(sel)} of {-(-w.d // 4096):,} 4096-blocks x {w.n} workers per round"
+        else:
+            d = min(w.d, blocks * 4096)
+            offs, gidx = None, None
+            self.sample = f"the first {d:,} coordinates x {w.n} workers per round"
+
+        def quant(s):
+            if offs is not None and s.kind in (W.Q_SIGN_L1, W.Q_UNIFORM_MAX):
+                o = offs
+            else:
+                o = O.group_offsets(d, s.group if 0 < s.group <= d else 0)
+            return O.Quantizer(s.kind, s.bits, o, stochastic=s.stochastic, pow2_k=s.pow2_k, pow2_K=s.pow2_K)
+
+        self.d, self.n = d, w.n
+        self.orc = O.OracleRound(d, w.n, quant(w.qw), quant(w.qs), w.alpha, w.beta1, w.beta2, w.eps,
+                                 seed=w.seed, mode=placement, gidx=gidx, threads=1)
+        rng = np.random.default_rng(0)
+        self.grads = [(rng.standard_normal(d) * w.grad_std).astype(np.float32) for _ in range(w.n)]
+        self.x = np.zeros(d, np.float32)
+
+    def step(self):
+        self.orc.compress_all(self.grads)
+        self.orc.server_step()
+        self.orc.apply(self.x)
+
+    @property
+    def units_per_step(self) -> int:
+        return self.n * self.d
+
+
+def cpu_baseline(w, placement: int, seconds: float = 12.0, blocks: int = 16):
+    """Oracle rounds on the sample, repeated for about `seconds` of CPU work."""
+    ob = OracleSample(w, placement, blocks)
+    rounds, t0 = 0, time.perf_counter()
+    while True:
+        ob.step()
+        rounds += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    return {"value": rounds * ob.units_per_step / el, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{ob.sample}; {rounds} rounds in {el:.1f} s, single-threaded C oracle"}
+
+
+# ---------------------------------------------------------------------------------- GPU bench
+
+def run_gpu(args, rank: int, world: int, local_rank: int):
+    import torch
+
+    import paper_2205_14473_gb300 as ea
+    from paper_2205_14473_gb300 import build as B
+    from paper_2205_14473_gb300 import workloads as W
+
+    B.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = _workload(args.workload)
+    placement = 0 if args.placement == "worker" else 1
+    cfg = ea.EAConfig.from_workload(w, placement=placement)
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        rnd = ea.EARound(cfg, stream=stream, device=dev)
+        grads = [torch.empty(w.d, dtype=torch.float32, device=dev) for _ in range(w.n)]
+        for i, g in enumerate(grads):
+            W.gradient_device(w, i, 0, g)
+        x = torch.zeros(w.d, dtype=torch.float32, device=dev)
+    stream.synchronize()
+
+    def one_round(events=None):
+        for i in range(w.n):
+            if events is not None:
+                events["c0"][i].record(stream)
+            rnd.worker_compress(i, grads[i])
+            if events is not None:
+                events["c1"][i].record(stream)
+        if events is not None:
+            events["s0"].record(stream)
+        rnd.server_step()
+        if events is not None:
+            events["s1"].record(stream)
+        rnd.apply(x)
+        if events is not None:
+            events["a1"].record(stream)
+
+    for _ in range(args.warmup):
+        one_round()
+    stream.synchronize()
+
+    def mk():
+        E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+        return {"c0": [E() for _ in range(w.n)], "c1": [E() for _ in range(w.n)], "s0": E(), "s1": E(), "a1": E()}
+
+    per_step = [mk() for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier = (lambda: torch.distributed.barrier()) if world > 1 else (lambda: None)
+    with ClockSampler(local_rank) as clk:
+        time.sleep(0.3)
+        barrier()
+        torch.cuda.synchronize(dev)
+        start.record(stream)
+        for k in range(args.steps):
+            one_round(per_step[k])
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier()
+    ms_total = start.elapsed_time(end)
+    comp = [ev["c0"][i].elapsed_time(ev["c1"][i]) for ev in per_step for i in range(w.n)]
+    serv = [ev["s0"].elapsed_time(ev["s1"]) for ev in per_step]
+    appl = [ev["s1"].elapsed_time(ev["a1"]) for ev in per_step]
+    rnd.sync()
+
+    # ---- end to end through the C-ABI with host buffers: H2D of every worker's gradient from pinned
+    # host memory, the round, D2H of x; copies overlap the previous worker's compress on a copy stream
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, w, rnd, x, dev, stream)
+
+    t_max = ms_total
+    if world > 1:
+        tt = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        t_max = float(tt.item())
+    units = w.n * w.d * args.steps * world
+    value = units / (t_max / 1e3)
+    ab = algorithmic_bytes(w, placement)
+    peak, peak_kind = _peaks()
+    comp_ms = statistics.mean(comp)
+    achieved = ab["compress"] / (comp_ms / 1e3) / 1e9
+    traffic = _ncu_traffic("worker_kernel", w.name, placement)
+    def launches(spec):  # one kernel, plus finalize + encode when the scale groups span tiles
+        has_scale = spec.kind in (W.Q_SIGN_L1, W.Q_UNIFORM_MAX)
+        one_pass = spec.group == 4096 or ((spec.group == 0 or spec.group >= w.d) and w.d <= 4096)
+        return 1 if (not has_scale or one_pass) else 3
+    launches_per_round = w.n * launches(w.qw) + launches(w.qs) + 1
+    rnd_ws = rnd.workspace_bytes
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": _describe(w, placement), "d": w.d, "n_workers": w.n, "global_batch": None,
+                   "seq_len": None, "parallelism": f"replicas{world}" if world > 1 else "single GPU",
+                   "l2": "inputs larger than L2 (working set %.0f GB)" % ((rnd_ws + (w.n + 1) * w.d * 4) / 1e9),
+                   "placement": "worker" if placement == 0 else "server"},
+        "roofline": {"bound": "hbm", "kernel": "worker_kernel (compress)", "achieved": achieved, "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak, "traffic": traffic,
+                     "algorithmic_bytes_per_launch": ab["compress"]},
+        "kernels_ms": {"compress_mean": comp_ms, "compress_min": min(comp), "server_mean": statistics.mean(serv),
+                       "apply_mean": statistics.mean(appl),
+                       "server_gbs": ab["server"] / (statistics.mean(serv) / 1e3) / 1e9,
+                       "apply_gbs": ab["apply"] / (statistics.mean(appl) / 1e3) / 1e9,
+                       "round_gbs": ab["round"] / (t_max / args.steps / 1e3) / 1e9},
+        "gpu_launches": launches_per_round * args.steps,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+    }
+    return out
+
+
+def run_e2e(args, w, rnd, x, dev, stream):
+    import torch
+
+    import paper_2205_14473_gb300 as ea
+
+    avail = 0
+    try:
+        for line in open("/proc/meminfo"):
+            if line.startswith("MemAvailable:"):
+                avail = int(line.split()[1]) * 1024
+    except Exception:
+        pass
+    gbytes = w.d * 4
+    n_host = w.n
+    while n_host > 1 and n_host * gbytes > 0.25 * avail:
+        n_host //= 2
+    host = [torch.empty(w.d, dtype=torch.float32, pin_memory=True) for _ in range(n_host)]
+    for i, h in enumerate(host):
+        h.normal_(0.0, w.grad_std)
+    x_host = torch.empty(w.d, dtype=torch.float32, pin_memory=True)
+    staging = [torch.empty(w.d, dtype=torch.float32, device=dev) for _ in range(2)]
+    copy = torch.cuda.Stream(dev)
+    ev_copied = [torch.cuda.Event() for _ in range(2)]
+    ev_used = [torch.cuda.Event() for _ in range(2)]
+
+    def step():
+        for i in range(w.n):
+            b = i % 2
+            with torch.cuda.stream(copy):
+                copy.wait_event(ev_used[b])
+                staging[b].copy_(host[i % n_host], non_blocking=True)
+                ev_copied[b].record(copy)
+            stream.wait_event(ev_copied[b])
+            ea.ea_worker_compress(rnd.h, i, staging[b].data_ptr())
+            ev_used[b].record(stream)
+        ea.ea_server_step(rnd.h)
+        ea.ea_worker_apply(rnd.h, x.data_ptr())
+        with torch.cuda.stream(stream):
+            x_host.copy_(x, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize(dev)
+    el = time.perf_counter() - t0
+    return {"value": w.n * w.d * args.steps / el, "unit": UNIT, "h2d_bytes_per_step": w.n * gbytes,
+            "d2h_bytes_per_step": gbytes, "ms_per_step": el / args.steps * 1e3,
+            "host_buffers": n_host,
+            "note": "ea_worker_compress/ea_server_step/ea_worker_apply with every gradient copied from pinned "
+                    "host memory (double-buffered on a copy stream) and x read back each step"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ea", choices=["ea", "reference"])
+    ap.add_argument("--workload", default="c5")
+    ap.add_argument("--placement", default="worker", choices=["worker", "server"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    w = _workload(args.workload)
+    placement = 0 if args.placement == "worker" else 1
+
+    if args.impl == "reference":
+        # the oracle on the host cores, same workload/metric; under torchrun only rank 0 runs
+        if rank != 0:
+            return
+        import oracle
+
+        oracle.build()
+        ob = OracleSample(w, placement, blocks=64)
+        for _ in range(args.warmup):
+            ob.step()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            ob.step()
+        el = time.perf_counter() - t0
+        val = args.steps * ob.units_per_step / el
+        cb = {"value": val, "unit": UNIT, "cores": 1, "kind": "oracle",
+              "sample": f"{ob.sample}; {args.steps} timed rounds in {el:.2f} s, single-threaded C oracle"}
+        out = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": 1,
+               "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+               "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+               "data": "synthetic", "config": {"workload": _describe(w, placement), "d": w.d, "n_workers": w.n},
+               "cpu_baseline": cb, "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0,
+                                           "d2h_bytes_per_step": 0}}
+        print(json.dumps(out), flush=True)
+        return
+
+    if world > 1:
+        import torch
+
+        torch.distributed.init_process_group("nccl")
+    out = run_gpu(args, rank, world, local_rank)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        oracle.build()
+        out["cpu_baseline"] = cpu_baseline(w, placement, seconds=args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch
+
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

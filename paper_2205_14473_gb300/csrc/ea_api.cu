@@ -1,0 +1,562 @@
+// ea_api.cu -- host side of the C ABI in include/ea.h: configuration checks, workspace layout,
+// the round protocol of Algorithms 1-2, kernel launches and the bits ledger of Corollary 1.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "ea.h"
+#include "ea_internal.h"
+
+using namespace ea;
+
+namespace {
+
+thread_local std::string g_last_error;  // failures that have no handle yet
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct QHost {
+    int kind = 0, bits = 0, stochastic = 0, k = 0, K = 0;
+    int gkind = GK_WHOLE, log2G = -1, pass = PASS_FUSED;
+    int64_t G = 0, n_groups = 1, n_words = 0, n_pairs = 0;
+    bool has_scales = false;
+    std::vector<int64_t> offsets;     // GK_SEG
+    std::vector<int32_t> tile_group;  // GK_SEG
+    std::vector<int64_t> pair_base;   // PASS_STASH
+    // device copies (inside the workspace)
+    int64_t *d_offsets = nullptr, *d_pair_base = nullptr;
+    int32_t *d_tile_group = nullptr;
+};
+
+// Sizes of every workspace buffer, in the order they are carved.
+struct Layout {
+    size_t e_w, m_w, v_w, e_s, m_s, v_s, codes_w, scales_w, codes_s, scales_s, partials;
+    size_t off_w, tg_w, pb_w, off_s, tg_s, pb_s;
+    int64_t dpad, wcode_stride, wscale_stride;
+};
+
+}  // namespace
+
+struct ea_handle {
+    ea_config cfg{};
+    QHost qw, qs;
+    Layout lay{};
+    cudaStream_t stream = nullptr;
+    int64_t n_tiles = 0;
+    float *m = nullptr, *v = nullptr, *e = nullptr, *es = nullptr, *ms = nullptr, *vs = nullptr;
+    uint32_t *wcodes = nullptr, *scodes = nullptr;
+    float *wscales = nullptr, *sscales = nullptr;
+    double *partials = nullptr;
+    Hyper hp{};
+    int64_t t = 0;
+    std::vector<unsigned char> compressed;
+    int n_compressed = 0;
+    bool has_message = false;
+    uint64_t up_bits = 0, down_bits = 0;
+    std::string err;
+};
+
+namespace {
+
+int fail(ea_handle *h, int code, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (h) h->err = buf;
+    else g_last_error = buf;
+    return code;
+}
+
+int check_cuda(ea_handle *h, cudaError_t e, const char *what)
+{
+    if (e == cudaSuccess) return EA_OK;
+    return fail(h, EA_E_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int ilog2_exact(int64_t x)
+{
+    if (x <= 0 || (x & (x - 1))) return -1;
+    int r = 0;
+    while ((int64_t{1} << r) < x) ++r;
+    return r;
+}
+
+// Validate one quantizer and derive its groups, tables and pass.
+int setup_quant(const ea_quantizer &q, int64_t d, const char *name, QHost &out)
+{
+    out = QHost{};
+    out.kind = q.kind;
+    out.bits = q.bits;
+    out.stochastic = q.stochastic;
+    out.k = q.pow2_k;
+    out.K = q.pow2_K;
+    switch (q.kind) {
+    case EA_Q_IDENTITY:
+        if (q.bits != 32) return fail(nullptr, EA_E_INVAL, "%s: the identity quantizer has 32 bits", name);
+        break;
+    case EA_Q_SIGN_L1:
+        if (q.bits != 1) return fail(nullptr, EA_E_INVAL, "%s: the scaled sign has 1 bit", name);
+        break;
+    case EA_Q_UNIFORM_MAX:
+        if (q.bits != 2 && q.bits != 4 && q.bits != 8 && q.bits != 16)
+            return fail(nullptr, EA_E_UNSUPPORTED, "%s: uniform grids of 2, 4, 8 or 16 bits only", name);
+        break;
+    case EA_Q_POW2:
+        if (q.bits != 4 && q.bits != 8)
+            return fail(nullptr, EA_E_UNSUPPORTED, "%s: power-of-two codes of 4 or 8 bits only", name);
+        if (q.pow2_k < -126 || q.pow2_K > 127 || q.pow2_k >= q.pow2_K)
+            return fail(nullptr, EA_E_INVAL, "%s: need -126 <= k < K <= 127", name);
+        if (static_cast<int64_t>(q.pow2_K) - q.pow2_k + 2 > (int64_t{1} << (q.bits - 1)))
+            return fail(nullptr, EA_E_INVAL, "%s: K - k + 1 levels and the zero code need more than %d bits",
+                        name, q.bits);
+        break;
+    default:
+        return fail(nullptr, EA_E_INVAL, "%s: unknown quantizer kind %d", name, q.kind);
+    }
+    if (q.stochastic != 0 && q.stochastic != 1) return fail(nullptr, EA_E_INVAL, "%s: stochastic is 0 or 1", name);
+    if (q.stochastic && q.kind != EA_Q_UNIFORM_MAX)
+        return fail(nullptr, EA_E_INVAL, "%s: stochastic rounding applies to the uniform grid only", name);
+    out.has_scales = q.kind == EA_Q_SIGN_L1 || q.kind == EA_Q_UNIFORM_MAX;
+    out.n_words = (d * q.bits + 31) / 32;
+
+    const int64_t n_tiles = (d + kTile - 1) / kTile;
+    if (!out.has_scales) {
+        out.gkind = GK_WHOLE;
+        out.n_groups = 0;
+        out.pass = PASS_FUSED;
+        return EA_OK;
+    }
+    if (q.group == 0) {
+        out.gkind = GK_WHOLE;
+        out.n_groups = 1;
+    } else if (q.group > 0) {
+        out.gkind = GK_BLOCK;
+        out.G = q.group;
+        out.log2G = ilog2_exact(q.group);
+        out.n_groups = (d + q.group - 1) / q.group;
+    } else {
+        if (!q.seg_lengths || q.n_seg < 1) return fail(nullptr, EA_E_INVAL, "%s: segments need lengths", name);
+        out.gkind = GK_SEG;
+        out.n_groups = q.n_seg;
+        out.offsets.resize(q.n_seg + 1);
+        out.offsets[0] = 0;
+        for (int i = 0; i < q.n_seg; ++i) {
+            if (q.seg_lengths[i] <= 0) return fail(nullptr, EA_E_INVAL, "%s: segment %d is empty", name, i);
+            out.offsets[i + 1] = out.offsets[i] + q.seg_lengths[i];
+        }
+        if (out.offsets.back() != d)
+            return fail(nullptr, EA_E_INVAL, "%s: segment lengths sum to %lld, not d = %lld", name,
+                        static_cast<long long>(out.offsets.back()), static_cast<long long>(d));
+        out.tile_group.resize(n_tiles);
+        int64_t gi = 0;
+        for (int64_t t = 0; t < n_tiles; ++t) {
+            while (out.offsets[gi + 1] <= t * kTile) ++gi;
+            out.tile_group[t] = static_cast<int32_t>(gi);
+        }
+    }
+    // One pass when every group is exactly one tile; otherwise partial norms per (tile, group).
+    const bool block_tiles = out.gkind == GK_BLOCK && out.G == kTile;
+    const bool single_tile = out.n_groups == 1 && d <= kTile;
+    if (block_tiles || single_tile) {
+        out.pass = PASS_FUSED;
+    } else {
+        out.pass = PASS_STASH;
+        out.pair_base.resize(out.n_groups + 1);
+        out.pair_base[0] = 0;
+        for (int64_t gi = 0; gi < out.n_groups; ++gi) {
+            int64_t b, e;
+            if (out.gkind == GK_WHOLE) { b = 0; e = d; }
+            else if (out.gkind == GK_BLOCK) { b = gi * out.G; e = std::min(d, (gi + 1) * out.G); }
+            else { b = out.offsets[gi]; e = out.offsets[gi + 1]; }
+            out.pair_base[gi + 1] = out.pair_base[gi] + ((e - 1) / kTile - b / kTile + 1);
+        }
+        out.n_pairs = out.pair_base.back();
+    }
+    return EA_OK;
+}
+
+int validate(const ea_config *cfg, QHost &qw, QHost &qs)
+{
+    if (!cfg) return fail(nullptr, EA_E_INVAL, "config is NULL");
+    if (cfg->d < 1) return fail(nullptr, EA_E_INVAL, "d must be >= 1");
+    if (cfg->d > (int64_t{1} << 40)) return fail(nullptr, EA_E_UNSUPPORTED, "d above 2^40");
+    if (cfg->n < 1 || cfg->n > 1024) return fail(nullptr, EA_E_INVAL, "n must be in [1, 1024]");
+    if (cfg->placement != EA_ADAM_AT_WORKER && cfg->placement != EA_ADAM_AT_SERVER)
+        return fail(nullptr, EA_E_INVAL, "unknown placement %d", cfg->placement);
+    if (cfg->error_feedback != 0 && cfg->error_feedback != 1)
+        return fail(nullptr, EA_E_INVAL, "error_feedback is 0 or 1");
+    if (cfg->reserved != 0) return fail(nullptr, EA_E_INVAL, "reserved must be 0");
+    if (!std::isfinite(cfg->alpha)) return fail(nullptr, EA_E_INVAL, "alpha must be finite");
+    if (!(cfg->beta1 >= 0.0f && cfg->beta1 < 1.0f)) return fail(nullptr, EA_E_INVAL, "beta1 must be in [0, 1)");
+    if (!(cfg->beta2 >= 0.0f && cfg->beta2 < 1.0f)) return fail(nullptr, EA_E_INVAL, "beta2 must be in [0, 1)");
+    if (!(cfg->eps > 0.0f) || !std::isfinite(cfg->eps)) return fail(nullptr, EA_E_INVAL, "eps (= v_0) must be > 0");
+    int r = setup_quant(cfg->qw, cfg->d, "Q_w", qw);
+    if (r != EA_OK) return r;
+    return setup_quant(cfg->qs, cfg->d, "Q_s", qs);
+}
+
+Layout make_layout(const ea_config &c, const QHost &qw, const QHost &qs)
+{
+    Layout L{};
+    const bool W = c.placement == EA_ADAM_AT_WORKER;
+    const int64_t n_tiles = (c.d + kTile - 1) / kTile;
+    L.dpad = static_cast<int64_t>(align_up(static_cast<size_t>(c.d), 64));
+    const size_t vec = static_cast<size_t>(L.dpad) * sizeof(float);
+    L.e_w = vec * c.n;
+    L.m_w = W ? vec * c.n : 0;
+    L.v_w = W ? vec * c.n : 0;
+    L.e_s = vec;
+    L.m_s = W ? 0 : vec;
+    L.v_s = W ? 0 : vec;
+    // code buffers padded to 256 bytes so that 8- and 16-byte code stores of the last slot stay inside
+    L.wcode_stride = static_cast<int64_t>(align_up(static_cast<size_t>(qw.n_words), 64));
+    L.wscale_stride = static_cast<int64_t>(align_up(static_cast<size_t>(std::max<int64_t>(qw.n_groups, 1)), 64));
+    L.codes_w = static_cast<size_t>(L.wcode_stride) * 4 * c.n;
+    L.scales_w = static_cast<size_t>(L.wscale_stride) * 4 * c.n;
+    L.codes_s = align_up(static_cast<size_t>(qs.n_words) * 4, kAlign);
+    L.scales_s = align_up(static_cast<size_t>(std::max<int64_t>(qs.n_groups, 1)) * 4, kAlign);
+    L.partials = static_cast<size_t>(std::max(qw.n_pairs, qs.n_pairs)) * sizeof(double);
+    L.off_w = qw.gkind == GK_SEG ? qw.offsets.size() * 8 : 0;
+    L.tg_w = qw.gkind == GK_SEG ? static_cast<size_t>(n_tiles) * 4 : 0;
+    L.pb_w = qw.pass == PASS_STASH ? qw.pair_base.size() * 8 : 0;
+    L.off_s = qs.gkind == GK_SEG ? qs.offsets.size() * 8 : 0;
+    L.tg_s = qs.gkind == GK_SEG ? static_cast<size_t>(n_tiles) * 4 : 0;
+    L.pb_s = qs.pass == PASS_STASH ? qs.pair_base.size() * 8 : 0;
+    return L;
+}
+
+size_t layout_bytes(const Layout &L)
+{
+    const size_t parts[] = {L.e_w, L.m_w, L.v_w, L.e_s, L.m_s, L.v_s, L.codes_w, L.scales_w, L.codes_s,
+                            L.scales_s, L.partials, L.off_w, L.tg_w, L.pb_w, L.off_s, L.tg_s, L.pb_s};
+    size_t total = 0;
+    for (size_t p : parts) total += align_up(p, kAlign);
+    return total;
+}
+
+Grouping device_grouping(const QHost &q)
+{
+    Grouping g{};
+    g.gkind = q.gkind;
+    g.log2G = q.log2G;
+    g.G = q.G;
+    g.n_groups = q.n_groups;
+    g.offsets = q.d_offsets;
+    g.tile_group = q.d_tile_group;
+    g.pair_base = q.d_pair_base;
+    return g;
+}
+
+QParams device_quant(const QHost &q)
+{
+    QParams p{};
+    p.kind = q.kind;  // the EA_Q_* and QK_* enumerators coincide
+    p.bits = q.bits;
+    p.stochastic = q.stochastic;
+    p.pow2_k = q.k;
+    p.pow2_K = q.K;
+    p.grp = device_grouping(q);
+    return p;
+}
+
+uint64_t message_bits(const QHost &q, int64_t d)
+{
+    return static_cast<uint64_t>(d) * static_cast<uint64_t>(q.bits) +
+           (q.has_scales ? 32ull * static_cast<uint64_t>(q.n_groups) : 0ull);
+}
+
+int check_dev_ptr(ea_handle *h, const void *p, const char *what)
+{
+    if (!p) return fail(h, EA_E_INVAL, "%s is NULL", what);
+    if (reinterpret_cast<uintptr_t>(p) % 16) return fail(h, EA_E_ALIGN, "%s is not 16-byte aligned", what);
+    return EA_OK;
+}
+
+// Finish a message whose scale groups span tiles: scales from the partial norms, then encode.
+int second_pass(ea_handle *h, const QHost &q, float *buf, uint32_t *words, float *scales, uint32_t id)
+{
+    FinalizeArgs f{};
+    f.d = h->cfg.d;
+    f.q = device_quant(q);
+    f.partials = h->partials;
+    f.scales = scales;
+    int r = check_cuda(h, launch_finalize(f, h->stream), "finalize launch");
+    if (r != EA_OK) return r;
+    EncodeArgs e{};
+    e.d = h->cfg.d;
+    e.n_tiles = h->n_tiles;
+    e.buf = buf;
+    e.q = device_quant(q);
+    e.words = words;
+    e.scales = scales;
+    e.ef = h->cfg.error_feedback;
+    e.seed = h->cfg.seed;
+    e.id = id;
+    e.t = static_cast<uint32_t>(h->t);
+    return check_cuda(h, launch_encode(e, h->stream), "encode launch");
+}
+
+}  // namespace
+
+extern "C" {
+
+int ea_workspace_bytes(const ea_config *cfg, size_t *bytes)
+{
+    QHost qw, qs;
+    if (!bytes) return fail(nullptr, EA_E_INVAL, "bytes is NULL");
+    const int r = validate(cfg, qw, qs);
+    if (r != EA_OK) return r;
+    *bytes = layout_bytes(make_layout(*cfg, qw, qs));
+    return EA_OK;
+}
+
+int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void *stream, ea_handle **out)
+{
+    if (!out) return fail(nullptr, EA_E_INVAL, "out is NULL");
+    *out = nullptr;
+    QHost qw, qs;
+    int r = validate(cfg, qw, qs);
+    if (r != EA_OK) return r;
+    const Layout L = make_layout(*cfg, qw, qs);
+    const size_t need = layout_bytes(L);
+    if (!workspace) return fail(nullptr, EA_E_WORKSPACE, "workspace is NULL");
+    if (reinterpret_cast<uintptr_t>(workspace) % kAlign)
+        return fail(nullptr, EA_E_WORKSPACE, "workspace is not 256-byte aligned");
+    if (workspace_bytes < need)
+        return fail(nullptr, EA_E_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, need);
+
+    ea_handle *h = new (std::nothrow) ea_handle;
+    if (!h) return fail(nullptr, EA_E_INVAL, "out of host memory");
+    h->cfg = *cfg;
+    h->cfg.qw.seg_lengths = nullptr;
+    h->cfg.qs.seg_lengths = nullptr;
+    h->qw = std::move(qw);
+    h->qs = std::move(qs);
+    h->lay = L;
+    h->stream = static_cast<cudaStream_t>(stream);
+    h->n_tiles = (cfg->d + kTile - 1) / kTile;
+    h->compressed.assign(cfg->n, 0);
+    h->hp.alpha = cfg->alpha;
+    h->hp.beta1 = cfg->beta1;
+    h->hp.beta2 = cfg->beta2;
+    h->hp.c1 = 1.0f - cfg->beta1;
+    h->hp.c2 = 1.0f - cfg->beta2;
+
+    char *p = static_cast<char *>(workspace);
+    auto take = [&p](size_t n) {
+        char *q = n ? p : nullptr;
+        p += align_up(n, kAlign);
+        return q;
+    };
+    h->e = reinterpret_cast<float *>(take(L.e_w));
+    h->m = reinterpret_cast<float *>(take(L.m_w));
+    h->v = reinterpret_cast<float *>(take(L.v_w));
+    h->es = reinterpret_cast<float *>(take(L.e_s));
+    h->ms = reinterpret_cast<float *>(take(L.m_s));
+    h->vs = reinterpret_cast<float *>(take(L.v_s));
+    h->wcodes = reinterpret_cast<uint32_t *>(take(L.codes_w));
+    h->wscales = reinterpret_cast<float *>(take(L.scales_w));
+    h->scodes = reinterpret_cast<uint32_t *>(take(L.codes_s));
+    h->sscales = reinterpret_cast<float *>(take(L.scales_s));
+    h->partials = reinterpret_cast<double *>(take(L.partials));
+    h->qw.d_offsets = reinterpret_cast<int64_t *>(take(L.off_w));
+    h->qw.d_tile_group = reinterpret_cast<int32_t *>(take(L.tg_w));
+    h->qw.d_pair_base = reinterpret_cast<int64_t *>(take(L.pb_w));
+    h->qs.d_offsets = reinterpret_cast<int64_t *>(take(L.off_s));
+    h->qs.d_tile_group = reinterpret_cast<int32_t *>(take(L.tg_s));
+    h->qs.d_pair_base = reinterpret_cast<int64_t *>(take(L.pb_s));
+
+    // Algorithm 2: m_0 = 0, v_0 = eps, e_1 = 0; Algorithm 1: e_1 = 0.  Messages start zeroed.
+    cudaStream_t s = h->stream;
+    r = check_cuda(h, cudaMemsetAsync(workspace, 0, need, s), "workspace clear");
+    if (r == EA_OK && cfg->placement == EA_ADAM_AT_WORKER)
+        r = check_cuda(h, launch_fill(h->v, static_cast<int64_t>(cfg->n) * L.dpad, cfg->eps, s), "v_0 fill");
+    if (r == EA_OK && cfg->placement == EA_ADAM_AT_SERVER)
+        r = check_cuda(h, launch_fill(h->vs, L.dpad, cfg->eps, s), "v_0 fill");
+    auto upload = [&](void *dst, const void *src, size_t n) {
+        if (r == EA_OK && n) r = check_cuda(h, cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s), "table upload");
+    };
+    upload(h->qw.d_offsets, h->qw.offsets.data(), L.off_w);
+    upload(h->qw.d_tile_group, h->qw.tile_group.data(), L.tg_w);
+    upload(h->qw.d_pair_base, h->qw.pair_base.data(), L.pb_w);
+    upload(h->qs.d_offsets, h->qs.offsets.data(), L.off_s);
+    upload(h->qs.d_tile_group, h->qs.tile_group.data(), L.tg_s);
+    upload(h->qs.d_pair_base, h->qs.pair_base.data(), L.pb_s);
+    if (r != EA_OK) {
+        g_last_error = h->err;
+        delete h;
+        return r;
+    }
+    *out = h;
+    return EA_OK;
+}
+
+int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
+{
+    if (!h) return fail(nullptr, EA_E_INVAL, "handle is NULL");
+    if (worker < 0 || worker >= h->cfg.n) return fail(h, EA_E_INVAL, "worker %d out of [0, %d)", worker, h->cfg.n);
+    int r = check_dev_ptr(h, g, "g");
+    if (r != EA_OK) return r;
+    if (h->compressed[worker])
+        return fail(h, EA_E_ORDER, "worker %d already compressed in round %lld", worker, static_cast<long long>(h->t));
+    const int64_t dp = h->lay.dpad;
+    WorkerArgs a{};
+    a.d = h->cfg.d;
+    a.n_tiles = h->n_tiles;
+    a.g = g;
+    const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
+    a.m = W ? h->m + worker * dp : nullptr;
+    a.v = W ? h->v + worker * dp : nullptr;
+    a.e = h->e + worker * dp;
+    a.q = device_quant(h->qw);
+    a.words = h->wcodes + worker * h->lay.wcode_stride;
+    a.scales = h->wscales + worker * h->lay.wscale_stride;
+    a.hp = h->hp;
+    a.ef = h->cfg.error_feedback;
+    a.pass = h->qw.pass;
+    a.seed = h->cfg.seed;
+    a.id = static_cast<uint32_t>(worker);
+    a.t = static_cast<uint32_t>(h->t);
+    a.partials = h->partials;
+    r = check_cuda(h, launch_worker(W ? MODE_W : MODE_S, a, h->stream), "worker launch");
+    if (r == EA_OK && h->qw.pass == PASS_STASH) r = second_pass(h, h->qw, a.e, a.words, a.scales, a.id);
+    if (r != EA_OK) return r;
+    h->compressed[worker] = 1;
+    ++h->n_compressed;
+    return EA_OK;
+}
+
+int ea_server_step(ea_handle *h)
+{
+    if (!h) return fail(nullptr, EA_E_INVAL, "handle is NULL");
+    if (h->n_compressed != h->cfg.n)
+        return fail(h, EA_E_ORDER, "round %lld: %d of %d workers compressed", static_cast<long long>(h->t),
+                    h->n_compressed, h->cfg.n);
+    ServerArgs a{};
+    a.d = h->cfg.d;
+    a.n_tiles = h->n_tiles;
+    a.n = h->cfg.n;
+    a.wwords = h->wcodes;
+    a.wwords_stride = h->lay.wcode_stride;
+    a.wscales = h->wscales;
+    a.wscales_stride = h->lay.wscale_stride;
+    a.qw = device_quant(h->qw);
+    a.qs = device_quant(h->qs);
+    a.words = h->scodes;
+    a.scales = h->sscales;
+    a.es = h->es;
+    a.ms = h->ms;
+    a.vs = h->vs;
+    a.hp = h->hp;
+    a.ef = h->cfg.error_feedback;
+    a.pass = h->qs.pass;
+    a.seed = h->cfg.seed;
+    a.t = static_cast<uint32_t>(h->t);
+    a.partials = h->partials;
+    const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
+    int r = check_cuda(h, W ? launch_server_w(a, h->stream) : launch_server_s(a, h->stream), "server launch");
+    if (r == EA_OK && h->qs.pass == PASS_STASH)
+        r = second_pass(h, h->qs, h->es, h->scodes, h->sscales, static_cast<uint32_t>(h->cfg.n));
+    if (r != EA_OK) return r;
+    h->up_bits += static_cast<uint64_t>(h->cfg.n) * message_bits(h->qw, h->cfg.d);
+    h->down_bits += static_cast<uint64_t>(h->cfg.n) * message_bits(h->qs, h->cfg.d);
+    ++h->t;
+    h->compressed.assign(h->cfg.n, 0);
+    h->n_compressed = 0;
+    h->has_message = true;
+    return EA_OK;
+}
+
+int ea_worker_apply(ea_handle *h, float *x)
+{
+    if (!h) return fail(nullptr, EA_E_INVAL, "handle is NULL");
+    int r = check_dev_ptr(h, x, "x");
+    if (r != EA_OK) return r;
+    if (!h->has_message) return fail(h, EA_E_ORDER, "no broadcast yet: call ea_server_step first");
+    ApplyArgs a{};
+    a.d = h->cfg.d;
+    a.x = x;
+    a.q = device_quant(h->qs);
+    a.words = h->scodes;
+    a.scales = h->sscales;
+    return check_cuda(h, launch_apply(a, h->stream), "apply launch");
+}
+
+int ea_bits_sent(const ea_handle *h, uint64_t *up_bits, uint64_t *down_bits)
+{
+    if (!h || !up_bits || !down_bits) return fail(nullptr, EA_E_INVAL, "NULL argument");
+    *up_bits = h->up_bits;
+    *down_bits = h->down_bits;
+    return EA_OK;
+}
+
+int ea_round_index(const ea_handle *h, int64_t *t)
+{
+    if (!h || !t) return fail(nullptr, EA_E_INVAL, "NULL argument");
+    *t = h->t;
+    return EA_OK;
+}
+
+int ea_get_view(const ea_handle *h, int32_t which, int32_t index, void **dev_ptr, size_t *bytes)
+{
+    if (!h || !dev_ptr || !bytes) return fail(nullptr, EA_E_INVAL, "NULL argument");
+    ea_handle *hm = const_cast<ea_handle *>(h);
+    const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
+    const bool per_worker = which == EA_VIEW_M || which == EA_VIEW_V || which == EA_VIEW_E_WORKER ||
+                            which == EA_VIEW_CODES_WORKER || which == EA_VIEW_SCALES_WORKER;
+    if (per_worker && (index < 0 || index >= h->cfg.n))
+        return fail(hm, EA_E_INVAL, "worker %d out of [0, %d)", index, h->cfg.n);
+    const int64_t dp = h->lay.dpad;
+    const size_t vec = static_cast<size_t>(h->cfg.d) * 4;
+    void *p = nullptr;
+    size_t n = 0;
+    switch (which) {
+    case EA_VIEW_M: if (W) { p = h->m + index * dp; n = vec; } break;
+    case EA_VIEW_V: if (W) { p = h->v + index * dp; n = vec; } break;
+    case EA_VIEW_E_WORKER: p = h->e + index * dp; n = vec; break;
+    case EA_VIEW_E_SERVER: p = h->es; n = vec; break;
+    case EA_VIEW_M_SERVER: if (!W) { p = h->ms; n = vec; } break;
+    case EA_VIEW_V_SERVER: if (!W) { p = h->vs; n = vec; } break;
+    case EA_VIEW_CODES_WORKER: p = h->wcodes + index * h->lay.wcode_stride; n = h->qw.n_words * 4; break;
+    case EA_VIEW_SCALES_WORKER: p = h->wscales + index * h->lay.wscale_stride; n = h->qw.n_groups * 4; break;
+    case EA_VIEW_CODES_SERVER: p = h->scodes; n = h->qs.n_words * 4; break;
+    case EA_VIEW_SCALES_SERVER: p = h->sscales; n = h->qs.n_groups * 4; break;
+    default: return fail(hm, EA_E_INVAL, "unknown view %d", which);
+    }
+    if (!p && !(which == EA_VIEW_SCALES_WORKER || which == EA_VIEW_SCALES_SERVER))
+        return fail(hm, EA_E_INVAL, "view %d does not exist in this placement", which);
+    *dev_ptr = p;
+    *bytes = n;
+    return EA_OK;
+}
+
+int ea_sync_status(ea_handle *h)
+{
+    if (!h) return fail(nullptr, EA_E_INVAL, "handle is NULL");
+    int r = check_cuda(h, cudaStreamSynchronize(h->stream), "stream synchronize");
+    if (r != EA_OK) return r;
+    return check_cuda(h, cudaGetLastError(), "pending error");
+}
+
+const char *ea_last_error(const ea_handle *h)
+{
+    return h ? h->err.c_str() : g_last_error.c_str();
+}
+
+int ea_destroy(ea_handle *h)
+{
+    delete h;
+    return EA_OK;
+}
+
+}  // extern "C"

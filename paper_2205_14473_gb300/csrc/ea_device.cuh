@@ -1,0 +1,367 @@
+// ea_device.cuh -- device building blocks of the round kernels: Philox4x32-10, the compensated
+// l1 reduction, the quantizers of Definition 1 / Examples 1-2 / Definition 3, code packing.
+//
+// Every per-coordinate expression uses the explicit round-to-nearest intrinsics (__fadd_rn,
+// __fmul_rn, __fdiv_rn, __fsqrt_rn), so nothing is contracted into an FMA and the order of
+// Algorithms 1-2 is kept: the result is the binary32 evaluation of the paper's expressions.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "ea_internal.h"
+
+namespace ea {
+
+// ------------------------------------------------------------------------------ Philox4x32-10
+// The counter-based generator of Salmon, Moraes, Dror and Shaw (SC'11): ten rounds of two 32x32
+// multiplies of the even words, the odd words and the key xored into the high halves, the key
+// advanced by the Weyl constants between rounds.  Coordinate j draws word j mod 4 of the counter
+// (j/4 low, j/4 high, id, round) under the key (seed low, seed high).
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k)
+{
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+        c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+        k.x += 0x9E3779B9u;
+        k.y += 0xBB67AE85u;
+    }
+    return c;
+}
+
+// The four uniform variates U in [0, 1) (24 bits) of coordinates j0 .. j0+3 (j0 % 4 == 0).
+__device__ __forceinline__ void uniforms4(uint64_t seed, uint32_t id, uint32_t t, int64_t j0, float U[4])
+{
+    const uint64_t blk = static_cast<uint64_t>(j0) >> 2;
+    const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(blk), static_cast<uint32_t>(blk >> 32), id, t),
+                                  make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32)));
+    U[0] = __fmul_rn(__uint2float_rn(w.x >> 8), 0x1p-24f);
+    U[1] = __fmul_rn(__uint2float_rn(w.y >> 8), 0x1p-24f);
+    U[2] = __fmul_rn(__uint2float_rn(w.z >> 8), 0x1p-24f);
+    U[3] = __fmul_rn(__uint2float_rn(w.w >> 8), 0x1p-24f);
+}
+
+// -------------------------------------------------------------------- compensated summation
+// Sums of |u| are carried as an unevaluated pair hi + lo of binary32 numbers: TwoSum keeps the
+// rounding error of every addition, so a 4096-term sum is accurate to ~2^-44 relative without the
+// (on this part, scarce) binary64 pipeline.  Only the CTA total is converted to binary64.
+struct DF {
+    float hi, lo;
+};
+
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &err)
+{
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    err = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+__device__ __forceinline__ DF df_add(DF a, DF b)
+{
+    float s, e;
+    two_sum(a.hi, b.hi, s, e);
+    float lo = __fadd_rn(__fadd_rn(a.lo, b.lo), e);
+    const float hi = __fadd_rn(s, lo);
+    lo = __fsub_rn(lo, __fsub_rn(hi, s));
+    return {hi, lo};
+}
+
+// Add x to an accumulator whose error terms are collected in acc.lo (Neumaier's form).
+__device__ __forceinline__ void df_accumulate(DF &acc, float x)
+{
+    float s, e;
+    two_sum(acc.hi, x, s, e);
+    acc.hi = s;
+    acc.lo = __fadd_rn(acc.lo, e);
+}
+
+// CTA-wide sum; every thread receives the same binary64 value (fixed combination order).
+__device__ __forceinline__ double block_sum(DF v, DF *red, double *bcast)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        DF w{__shfl_down_sync(0xffffffffu, v.hi, o), __shfl_down_sync(0xffffffffu, v.lo, o)};
+        v = df_add(v, w);
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        DF t = red[0];
+#pragma unroll
+        for (int w = 1; w < kWarps; ++w) t = df_add(t, red[w]);
+        *bcast = static_cast<double>(t.hi) + static_cast<double>(t.lo);
+    }
+    __syncthreads();
+    return *bcast;
+}
+
+// CTA-wide maximum of non-negative values (exact: compares bit patterns).
+__device__ __forceinline__ float block_max(float a, uint32_t *red, float *bcast)
+{
+    const uint32_t b = __reduce_max_sync(0xffffffffu, __float_as_uint(a));
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) red[warp] = b;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t m = red[0];
+#pragma unroll
+        for (int w = 1; w < kWarps; ++w) m = max(m, red[w]);
+        *bcast = __uint_as_float(m);
+    }
+    __syncthreads();
+    return *bcast;
+}
+
+// Group scale of the scaled sign: ||u||_1 / G, the division in binary64, one rounding to binary32.
+__device__ __forceinline__ float sign_scale(double l1, int64_t len)
+{
+    return len > 0 ? __double2float_rn(__ddiv_rn(l1, static_cast<double>(len))) : 0.0f;
+}
+
+// ------------------------------------------------------------------------------- quantizers
+// Codes: sign 1 = (u >= 0); uniform q + L with L = 2^(b-1) - 1; pow2 sign bit b-1 and exponent
+// index below it, all-ones index = 0; identity = the binary32 pattern.
+
+__device__ __forceinline__ int unif_L(int bits) { return (1 << (bits - 1)) - 1; }
+
+// Example 1: z = u / s, y = z L, nearest grid index (ties to even) or stochastic rounding.
+__device__ __forceinline__ int unif_index(float u, float s, float Lf, bool stochastic, float U)
+{
+    if (!(s > 0.0f)) return 0;
+    const float z = __fdiv_rn(u, s);
+    const float y = __fmul_rn(z, Lf);
+    if (stochastic) {
+        const float f = floorf(y);
+        const float frac = __fsub_rn(y, f);
+        return static_cast<int>(f) + (U < frac ? 1 : 0);
+    }
+    return __float2int_rn(y);
+}
+
+// Example 2: the nearest of {2^k, ..., 2^K} to |u| (ties up), read off the binary32 exponent.
+__device__ __forceinline__ uint32_t pow2_code(float u, int k, int K, int bits)
+{
+    const uint32_t zero_idx = (1u << (bits - 1)) - 1u;
+    if (u == 0.0f) return zero_idx;
+    const uint32_t ub = __float_as_uint(u);
+    const uint32_t sign = (ub >> 31) << (bits - 1);
+    const uint32_t ab = ub & 0x7fffffffu;
+    const uint32_t lo_b = static_cast<uint32_t>(k + 127) << 23, hi_b = static_cast<uint32_t>(K + 127) << 23;
+    int j;
+    if (ab <= lo_b) j = k;
+    else if (ab >= hi_b) j = K;
+    else j = static_cast<int>(ab >> 23) - 127 + ((ab & 0x400000u) ? 1 : 0);  // mantissa >= 1.5 goes up
+    return sign | static_cast<uint32_t>(j - k);
+}
+
+__device__ __forceinline__ float pow2_value(uint32_t code, int k, int bits)
+{
+    const uint32_t zero_idx = (1u << (bits - 1)) - 1u;
+    const uint32_t idx = code & zero_idx;
+    if (idx == zero_idx) return 0.0f;
+    const float mag = __uint_as_float(static_cast<uint32_t>(k + static_cast<int>(idx) + 127) << 23);
+    return (code >> (bits - 1)) ? -mag : mag;
+}
+
+// Encode one coordinate, returning the code and the decoded value Q(u).
+template <int QK>
+__device__ __forceinline__ uint32_t encode1(float u, float s, const QParams &q, float Lf, int L, float U, float &dec)
+{
+    if constexpr (QK == QK_SIGN) {
+        const bool pos = u >= 0.0f;
+        dec = pos ? s : -s;
+        return pos ? 1u : 0u;
+    } else if constexpr (QK == QK_UNIF) {
+        const int qi = unif_index(u, s, Lf, q.stochastic != 0, U);
+        dec = __fmul_rn(s, __fdiv_rn(static_cast<float>(qi), Lf));
+        return static_cast<uint32_t>(qi + L);
+    } else if constexpr (QK == QK_POW2) {
+        const uint32_t c = pow2_code(u, q.pow2_k, q.pow2_K, q.bits);
+        dec = pow2_value(c, q.pow2_k, q.bits);
+        return c;
+    } else {
+        dec = u;
+        return __float_as_uint(u);
+    }
+}
+
+// Decode one coordinate of a received message.  utab (may be null) holds fl(i / L), i = -L..L.
+template <int QK>
+__device__ __forceinline__ float decode1(uint32_t code, float s, const QParams &q, float Lf, int L, const float *utab)
+{
+    if constexpr (QK == QK_SIGN) {
+        return code ? s : -s;
+    } else if constexpr (QK == QK_UNIF) {
+        const float r = utab ? utab[code] : __fdiv_rn(static_cast<float>(static_cast<int>(code) - L), Lf);
+        return __fmul_rn(s, r);
+    } else if constexpr (QK == QK_POW2) {
+        return pow2_value(code, q.pow2_k, q.bits);
+    } else {
+        return __uint_as_float(code);
+    }
+}
+
+template <int QK>
+__device__ __forceinline__ constexpr bool has_scale()
+{
+    return QK == QK_SIGN || QK == QK_UNIF;
+}
+
+// ----------------------------------------------------------------------------- scale groups
+
+__device__ __forceinline__ int64_t group_begin(const Grouping &g, int64_t gi, int64_t d)
+{
+    if (g.gkind == GK_WHOLE) return 0;
+    if (g.gkind == GK_BLOCK) return gi * g.G;
+    return g.offsets[gi];
+}
+
+__device__ __forceinline__ int64_t group_end(const Grouping &g, int64_t gi, int64_t d)
+{
+    if (g.gkind == GK_WHOLE) return d;
+    if (g.gkind == GK_BLOCK) return min((gi + 1) * g.G, d);
+    return g.offsets[gi + 1];
+}
+
+// Group of coordinate j; `hint` must be a group index <= the answer (used for segments).
+__device__ __forceinline__ int64_t group_of(const Grouping &g, int64_t j, int64_t hint)
+{
+    if (g.gkind == GK_WHOLE) return 0;
+    if (g.gkind == GK_BLOCK) return g.log2G >= 0 ? (j >> g.log2G) : j / g.G;
+    int64_t gi = hint;
+    while (g.offsets[gi + 1] <= j) ++gi;
+    return gi;
+}
+
+__device__ __forceinline__ int64_t first_group_of_tile(const Grouping &g, int64_t tile)
+{
+    if (g.gkind == GK_WHOLE) return 0;
+    if (g.gkind == GK_BLOCK) return (tile * kTile) / g.G;
+    return g.tile_group[tile];
+}
+
+// --------------------------------------------------------------------------------- packing
+// Coordinate j's b-bit code sits at bit j*b of the little-endian word stream.  A float4 slot q
+// (coordinates 4q .. 4q+3) spans 4b bits, so for b <= 8 it lies inside word (q*b)/8.
+
+// Load the four codes of slot q.
+__device__ __forceinline__ void load_codes4(const uint32_t *__restrict__ words, int64_t q, int bits, uint32_t c[4])
+{
+    if (bits <= 8) {
+        const uint32_t w = __ldg(words + ((q * bits) >> 3));
+        const int sh = static_cast<int>((q * bits) & 7) * 4;
+        const uint32_t mask = (1u << bits) - 1u;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) c[i] = (w >> (sh + i * bits)) & mask;
+    } else if (bits == 16) {
+        const uint2 w = __ldg(reinterpret_cast<const uint2 *>(words) + q);
+        c[0] = w.x & 0xffffu;
+        c[1] = w.x >> 16;
+        c[2] = w.y & 0xffffu;
+        c[3] = w.y >> 16;
+    } else {
+        const uint4 w = __ldg(reinterpret_cast<const uint4 *>(words) + q);
+        c[0] = w.x;
+        c[1] = w.y;
+        c[2] = w.z;
+        c[3] = w.w;
+    }
+}
+
+// Spread the 8 bits of x to bit positions 0, 4, 8, ..., 28.
+__device__ __forceinline__ uint32_t spread8_by4(uint32_t x)
+{
+    x &= 0xffu;
+    x = (x | (x << 12)) & 0x000f000fu;
+    x = (x | (x << 6)) & 0x03030303u;
+    x = (x | (x << 3)) & 0x11111111u;
+    return x;
+}
+
+// Store the four codes of slot q (the same slot index on every lane is q_lane0 + lane).  Must be
+// called by all 32 lanes of the warp.  Codes of coordinates >= d are 0 (caller's job).
+// b = 1: one ballot per component; lanes 8g .. 8g+7 fill word (q_lane0 / 8) + g, whose bit
+// 4l + c is component c of lane 8g + l.
+__device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64_t q, int bits, const uint32_t c[4],
+                                             int64_t n_words)
+{
+    const int lane = threadIdx.x & 31;
+    if (bits == 1) {
+        const uint32_t b0 = __ballot_sync(0xffffffffu, c[0] != 0);
+        const uint32_t b1 = __ballot_sync(0xffffffffu, c[1] != 0);
+        const uint32_t b2 = __ballot_sync(0xffffffffu, c[2] != 0);
+        const uint32_t b3 = __ballot_sync(0xffffffffu, c[3] != 0);
+        if (lane < 4) {
+            const int sh = 8 * lane;
+            const uint32_t w = spread8_by4(b0 >> sh) | (spread8_by4(b1 >> sh) << 1) | (spread8_by4(b2 >> sh) << 2) |
+                               (spread8_by4(b3 >> sh) << 3);
+            const int64_t wi = ((q - lane) >> 3) + lane;  // q - lane is lane 0's slot
+            if (wi < n_words) words[wi] = w;
+        }
+    } else if (bits <= 8) {
+        uint32_t v = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v |= c[i] << (i * bits);
+        const int per_word = 8 / bits;             // slots per word: 4 (b=2), 2 (b=4), 1 (b=8)
+        const int pos = static_cast<int>(q & (per_word - 1));
+        v <<= pos * 4 * bits;
+        if (per_word >= 2) v |= __shfl_xor_sync(0xffffffffu, v, 1);
+        if (per_word >= 4) v |= __shfl_xor_sync(0xffffffffu, v, 2);
+        const int64_t wi = (q * bits) >> 3;
+        if (pos == 0 && wi < n_words) words[wi] = v;
+    } else if (bits == 16) {
+        if (2 * q < n_words)
+            reinterpret_cast<uint2 *>(words)[q] = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
+    } else {
+        if (4 * q < n_words) reinterpret_cast<uint4 *>(words)[q] = make_uint4(c[0], c[1], c[2], c[3]);
+    }
+}
+
+// The paper's Adam moment update and step (Algorithm 2): no bias correction, eps only as v_0.
+__device__ __forceinline__ float adam_step(float g, float &m, float &v, const Hyper &h)
+{
+    v = __fadd_rn(__fmul_rn(h.beta2, v), __fmul_rn(h.c2, __fmul_rn(g, g)));
+    m = __fadd_rn(__fmul_rn(h.beta1, m), __fmul_rn(h.c1, g));
+    return __fdiv_rn(__fmul_rn(h.alpha, m), __fsqrt_rn(v));
+}
+
+// ------------------------------------------------------------------------ vector helpers
+
+__device__ __forceinline__ void to_arr(const float4 &v, float a[4])
+{
+    a[0] = v.x;
+    a[1] = v.y;
+    a[2] = v.z;
+    a[3] = v.w;
+}
+
+__device__ __forceinline__ float4 to_f4(const float a[4]) { return make_float4(a[0], a[1], a[2], a[3]); }
+
+// Load slot q of p (4 coordinates from 4q) into a; coordinates >= d read as 0.
+__device__ __forceinline__ void load4(const float *__restrict__ p, int64_t q, int64_t d, float a[4])
+{
+    const int64_t j0 = 4 * q;
+    if (j0 + 4 <= d) {
+        to_arr(__ldcs(reinterpret_cast<const float4 *>(p) + q), a);
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) a[i] = (j0 + i < d) ? p[j0 + i] : 0.0f;
+    }
+}
+
+__device__ __forceinline__ void store4(float *__restrict__ p, int64_t q, int64_t d, const float a[4])
+{
+    const int64_t j0 = 4 * q;
+    if (j0 + 4 <= d) {
+        __stcs(reinterpret_cast<float4 *>(p) + q, to_f4(a));
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (j0 + i < d) p[j0 + i] = a[i];
+    }
+}
+
+}  // namespace ea

@@ -1,0 +1,115 @@
+// ea_internal.h -- launch parameters shared by the host API (ea_api.cu) and the kernel units.
+// Not installed; the public interface is include/ea.h.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace ea {
+
+// One CTA tile: 256 threads x 4 float4 slots = 4096 coordinates.  Tiles are aligned to multiples
+// of 4096 in the flat vector, so for every code width b a tile owns whole 32-bit code words.
+constexpr int kThreads = 256;
+constexpr int kSlots = 4;
+constexpr int kTile = kThreads * kSlots * 4;
+constexpr int kWarps = kThreads / 32;
+
+enum QKind : int { QK_IDENT = 0, QK_SIGN = 1, QK_UNIF = 2, QK_POW2 = 3 };
+enum GKind : int { GK_WHOLE = 0, GK_BLOCK = 1, GK_SEG = 2 };
+enum Mode : int { MODE_W = 0, MODE_S = 1 };  // Adam at the workers (the paper) / at the server
+
+// How a message's scale groups tile the vector.
+struct Grouping {
+    int gkind;
+    int log2G;                  // GK_BLOCK: log2 of G when G is a power of two, else -1
+    int64_t G;                  // GK_BLOCK: block length
+    int64_t n_groups;
+    const int64_t *offsets;     // GK_SEG: n_groups + 1 offsets (device)
+    const int32_t *tile_group;  // GK_SEG: first group that intersects each 4096-tile (device)
+    const int64_t *pair_base;   // n_groups + 1: first partial-sum slot of each group (device)
+};
+
+struct QParams {
+    int kind, bits, stochastic, pow2_k, pow2_K;
+    Grouping grp;
+};
+
+struct Hyper {
+    float alpha, beta1, beta2, c1, c2;  // c1 = 1 - beta1, c2 = 1 - beta2, rounded to binary32
+};
+
+// How the scale of a message is formed.
+enum Pass : int {
+    PASS_FUSED = 0,  // every group lies inside one tile: reduce, encode and store in one pass
+    PASS_STASH = 1   // groups span tiles: store the input in the residual buffer plus one
+                     // partial norm per (tile, group); finalize_kernel and encode_kernel finish
+};
+
+struct WorkerArgs {
+    int64_t d, n_tiles;
+    const float *g;
+    float *m, *v, *e;
+    QParams q;
+    uint32_t *words;
+    float *scales;
+    Hyper hp;
+    int ef, pass;
+    uint64_t seed;
+    uint32_t id, t;
+    double *partials;
+};
+
+struct ServerArgs {
+    int64_t d, n_tiles;
+    int n;
+    const uint32_t *wwords;   // worker i's codes at wwords + i * wwords_stride
+    int64_t wwords_stride;
+    const float *wscales;     // worker i's scales at wscales + i * wscales_stride
+    int64_t wscales_stride;
+    QParams qw, qs;
+    uint32_t *words;          // the broadcast
+    float *scales;
+    float *es, *ms, *vs;
+    Hyper hp;
+    int ef, pass;
+    uint64_t seed;
+    uint32_t t;
+    double *partials;
+};
+
+// Second pass of PASS_STASH: encode the stashed input in buf, leave the residual in buf.
+struct EncodeArgs {
+    int64_t d, n_tiles;
+    float *buf;
+    QParams q;
+    uint32_t *words;
+    const float *scales;
+    int ef;
+    uint64_t seed;
+    uint32_t id, t;
+};
+
+struct FinalizeArgs {
+    int64_t d;
+    QParams q;
+    const double *partials;
+    float *scales;
+};
+
+struct ApplyArgs {
+    int64_t d;
+    float *x;
+    QParams q;
+    const uint32_t *words;
+    const float *scales;
+};
+
+cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s);
+cudaError_t launch_server_w(const ServerArgs &a, cudaStream_t s);
+cudaError_t launch_server_s(const ServerArgs &a, cudaStream_t s);
+cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s);
+cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s);
+cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s);
+cudaError_t launch_fill(float *p, int64_t count, float value, cudaStream_t s);
+
+}  // namespace ea

@@ -1,0 +1,126 @@
+// ea_tile.cuh -- the common end of a worker or server tile: given the residual-corrected input u
+// of the tile's 4096 coordinates (held in registers, 16 per thread), form the group scale, encode
+// and pack the message, and keep the residual e = u - Q(u) (Algorithm 1 / Algorithm 2).
+#pragma once
+
+#include "ea_device.cuh"
+
+namespace ea {
+
+struct TileSmem {
+    DF red[kWarps];
+    uint32_t redm[kWarps];
+    double bcast;
+    float bcastf;
+};
+
+// Slot k of this thread in tile `tile`: coordinates 4q .. 4q+3.  Consecutive threads own
+// consecutive float4 slots, so every warp access is one contiguous 512-byte segment.
+__device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
+{
+    return tile * (kTile / 4) + k * kThreads + threadIdx.x;
+}
+
+// Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
+template <int QK>
+__device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
+                                             const QParams &q, uint32_t *words, float *resid, int ef,
+                                             uint64_t seed, uint32_t id, uint32_t t)
+{
+    const int L = (QK == QK_UNIF) ? unif_L(q.bits) : 0;
+    const float Lf = static_cast<float>(L);
+    const int64_t n_words = (d * q.bits + 31) >> 5;
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t qs = slot_of(tile, k);
+        const int64_t j0 = 4 * qs;
+        float U[4] = {0.f, 0.f, 0.f, 0.f};
+        if (QK == QK_UNIF && q.stochastic && j0 < d) uniforms4(seed, id, t, j0, U);
+        uint32_t c[4];
+        float e[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float dec = 0.0f;
+            c[i] = (j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec) : 0u;
+            e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;
+        }
+        store_codes4(words, qs, q.bits, c, n_words);
+        if (ef && j0 < d) store4(resid, qs, d, e);
+    }
+}
+
+// The tile's end for a quantizer with scale groups.
+//   PASS_FUSED: the tile is exactly one scale group (blocks of 4096): reduce, encode, store.
+//   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
+template <int QK>
+__device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile, int64_t d, const QParams &q,
+                                            uint32_t *words, float *scales, float *resid, int ef, int pass,
+                                            uint64_t seed, uint32_t id, uint32_t t, double *partials,
+                                            TileSmem &sm)
+{
+    if constexpr (!has_scale<QK>()) {
+        encode_store<QK>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t);
+        return;
+    } else {
+        const int64_t tile_lo = tile * kTile;
+        const int64_t tile_hi = min(tile_lo + static_cast<int64_t>(kTile), d);
+        if (pass == PASS_FUSED) {
+            float s;
+            if constexpr (QK == QK_SIGN) {
+                DF acc{0.0f, 0.0f};
+#pragma unroll
+                for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) df_accumulate(acc, fabsf(u[k][i]));  // invalid u are 0
+                s = sign_scale(block_sum(acc, sm.red, &sm.bcast), tile_hi - tile_lo);
+            } else {
+                float mx = 0.0f;
+#pragma unroll
+                for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) mx = fmaxf(mx, fabsf(u[k][i]));
+                s = block_max(mx, sm.redm, &sm.bcastf);
+            }
+            if (threadIdx.x == 0) scales[tile] = s;
+            encode_store<QK>(u, s, tile, d, q, words, resid, ef, seed, id, t);
+            return;
+        }
+        // PASS_STASH
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            const int64_t qs = slot_of(tile, k);
+            if (4 * qs < d) store4(resid, qs, d, u[k]);
+        }
+        const Grouping &G = q.grp;
+        for (int64_t gi = first_group_of_tile(G, tile);; ++gi) {
+            const int64_t gb = group_begin(G, gi, d), ge = group_end(G, gi, d);
+            const int64_t lo = max(gb, tile_lo), hi = min(ge, tile_hi);
+            double part;
+            if constexpr (QK == QK_SIGN) {
+                DF acc{0.0f, 0.0f};
+#pragma unroll
+                for (int k = 0; k < kSlots; ++k) {
+                    const int64_t j0 = 4 * slot_of(tile, k);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if (j0 + i >= lo && j0 + i < hi) df_accumulate(acc, fabsf(u[k][i]));
+                }
+                part = block_sum(acc, sm.red, &sm.bcast);
+            } else {
+                float mx = 0.0f;
+#pragma unroll
+                for (int k = 0; k < kSlots; ++k) {
+                    const int64_t j0 = 4 * slot_of(tile, k);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if (j0 + i >= lo && j0 + i < hi) mx = fmaxf(mx, fabsf(u[k][i]));
+                }
+                part = static_cast<double>(block_max(mx, sm.redm, &sm.bcastf));
+            }
+            if (threadIdx.x == 0) partials[G.pair_base[gi] + (tile - gb / kTile)] = part;
+            if (ge >= tile_hi) break;
+        }
+    }
+}
+
+}  // namespace ea

@@ -1,0 +1,205 @@
+// ea_worker.cu -- worker compress (Algorithm 2), the two-pass scale kernels, and x <- x - Q_s(w).
+#include "ea_tile.cuh"
+
+namespace ea {
+
+// Algorithm 2 for one worker on one 4096-coordinate tile.  With Adam at the worker:
+//   v <- beta2 v + (1-beta2) g^2, m <- beta1 m + (1-beta1) g, u = alpha m / sqrt(v) + e;
+// with Adam at the server: u = g + e.  Then Q_w(u) and e <- u - Q_w(u) (finish_tile).
+// HBM traffic per coordinate: 16 B read + 12 B written + b/8 B of code (Adam at the worker).
+template <int MODE, int QK>
+__global__ void __launch_bounds__(kThreads, 2) worker_kernel(const WorkerArgs a)
+{
+    __shared__ TileSmem sm;
+    const int64_t tile = blockIdx.x;
+    const int64_t d = a.d;
+
+    float g[kSlots][4], e[kSlots][4], m[kSlots][4], v[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        load4(a.g, q, d, g[k]);
+        load4(a.e, q, d, e[k]);
+        if (MODE == MODE_W) {
+            load4(a.m, q, d, m[k]);
+            load4(a.v, q, d, v[k]);
+        }
+    }
+    float u[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        const int64_t j0 = 4 * q;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float step = g[k][i];
+            if (MODE == MODE_W) step = adam_step(g[k][i], m[k][i], v[k][i], a.hp);
+            u[k][i] = (j0 + i < d) ? __fadd_rn(step, e[k][i]) : 0.0f;
+        }
+        if (MODE == MODE_W && j0 < d) {
+            store4(a.m, q, d, m[k]);
+            store4(a.v, q, d, v[k]);
+        }
+    }
+    finish_tile<QK>(u, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t, a.partials, sm);
+}
+
+// Second pass, one CTA per scale group: combine the group's per-tile partial norms in a fixed
+// order and write the group scale (Example 1: ||.||_inf; scaled sign: ||.||_1 / |group|).
+template <int QK>
+__global__ void __launch_bounds__(kThreads) finalize_kernel(const FinalizeArgs a)
+{
+    __shared__ double red[kWarps];
+    const int64_t gi = blockIdx.x;
+    const int64_t pb = a.q.grp.pair_base[gi], pe = a.q.grp.pair_base[gi + 1];
+    double acc = 0.0;
+    for (int64_t p = pb + threadIdx.x; p < pe; p += kThreads)
+        acc = (QK == QK_SIGN) ? __dadd_rn(acc, a.partials[p]) : fmax(acc, a.partials[p]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const double w = __shfl_down_sync(0xffffffffu, acc, o);
+        acc = (QK == QK_SIGN) ? __dadd_rn(acc, w) : fmax(acc, w);
+    }
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = red[0];
+        for (int w = 1; w < kWarps; ++w) t = (QK == QK_SIGN) ? __dadd_rn(t, red[w]) : fmax(t, red[w]);
+        const int64_t len = group_end(a.q.grp, gi, a.d) - group_begin(a.q.grp, gi, a.d);
+        a.scales[gi] = (QK == QK_SIGN) ? sign_scale(t, len) : static_cast<float>(t);
+    }
+}
+
+// Second pass, one CTA per tile: encode the stashed input with its group's scale and leave the
+// residual u - Q(u) in its place.
+template <int QK>
+__global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
+{
+    const int64_t tile = blockIdx.x;
+    const int64_t d = a.d;
+    const Grouping &G = a.q.grp;
+    const int L = (QK == QK_UNIF) ? unif_L(a.q.bits) : 0;
+    const float Lf = static_cast<float>(L);
+    const int64_t n_words = (d * a.q.bits + 31) >> 5;
+    const int64_t hint = first_group_of_tile(G, tile);
+    float u[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) load4(a.buf, slot_of(tile, k), d, u[k]);
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t qs = slot_of(tile, k);
+        const int64_t j0 = 4 * qs;
+        float U[4] = {0.f, 0.f, 0.f, 0.f};
+        if (QK == QK_UNIF && a.q.stochastic && j0 < d) uniforms4(a.seed, a.id, a.t, j0, U);
+        uint32_t c[4];
+        float e[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float dec = 0.0f;
+            c[i] = 0u;
+            if (j0 + i < d) {
+                const float s = a.scales[group_of(G, j0 + i, hint)];
+                c[i] = encode1<QK>(u[k][i], s, a.q, Lf, L, U[i], dec);
+            }
+            e[i] = a.ef ? __fsub_rn(u[k][i], dec) : 0.0f;
+        }
+        store_codes4(a.words, qs, a.q.bits, c, n_words);
+        if (j0 < d) store4(a.buf, qs, d, e);
+    }
+}
+
+// x <- x - Q_s(w): decode the broadcast and update x (Algorithm 1 and Algorithm 2).
+// HBM traffic per coordinate: 4 B read + 4 B written + b/8 B of code.
+template <int QK>
+__global__ void __launch_bounds__(kThreads) apply_kernel(const ApplyArgs a)
+{
+    const int64_t d = a.d;
+    const int64_t n_slots = (d + 3) >> 2;
+    const Grouping &G = a.q.grp;
+    const int L = (QK == QK_UNIF) ? unif_L(a.q.bits) : 0;
+    const float Lf = static_cast<float>(L);
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; q < n_slots;
+         q += static_cast<int64_t>(gridDim.x) * kThreads) {
+        const int64_t j0 = 4 * q;
+        float x[4];
+        load4(a.x, q, d, x);
+        uint32_t c[4];
+        load_codes4(a.words, q, a.q.bits, c);
+        const int64_t hint = first_group_of_tile(G, j0 / kTile);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (j0 + i < d) {
+                const float s = has_scale<QK>() ? a.scales[group_of(G, j0 + i, hint)] : 0.0f;
+                x[i] = __fsub_rn(x[i], decode1<QK>(c[i], s, a.q, Lf, L, nullptr));
+            }
+        }
+        store4(a.x, q, d, x);
+    }
+}
+
+__global__ void fill_kernel(float *p, int64_t count, float value)
+{
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < count;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        p[i] = value;
+}
+
+// ------------------------------------------------------------------------------- launchers
+
+template <int MODE>
+static cudaError_t launch_worker_mode(const WorkerArgs &a, cudaStream_t s)
+{
+    const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
+    switch (a.q.kind) {
+    case QK_SIGN: worker_kernel<MODE, QK_SIGN><<<grid, block, 0, s>>>(a); break;
+    case QK_UNIF: worker_kernel<MODE, QK_UNIF><<<grid, block, 0, s>>>(a); break;
+    case QK_POW2: worker_kernel<MODE, QK_POW2><<<grid, block, 0, s>>>(a); break;
+    default: worker_kernel<MODE, QK_IDENT><<<grid, block, 0, s>>>(a); break;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s)
+{
+    return mode == MODE_W ? launch_worker_mode<MODE_W>(a, s) : launch_worker_mode<MODE_S>(a, s);
+}
+
+cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s)
+{
+    const dim3 grid(static_cast<unsigned>(a.q.grp.n_groups)), block(kThreads);
+    if (a.q.kind == QK_SIGN) finalize_kernel<QK_SIGN><<<grid, block, 0, s>>>(a);
+    else finalize_kernel<QK_UNIF><<<grid, block, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s)
+{
+    const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
+    if (a.q.kind == QK_SIGN) encode_kernel<QK_SIGN><<<grid, block, 0, s>>>(a);
+    else encode_kernel<QK_UNIF><<<grid, block, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s)
+{
+    const int64_t n_slots = (a.d + 3) >> 2;
+    const int64_t want = (n_slots + kThreads - 1) / kThreads;
+    const dim3 grid(static_cast<unsigned>(want < 152 * 32 ? want : 152 * 32)), block(kThreads);
+    switch (a.q.kind) {
+    case QK_SIGN: apply_kernel<QK_SIGN><<<grid, block, 0, s>>>(a); break;
+    case QK_UNIF: apply_kernel<QK_UNIF><<<grid, block, 0, s>>>(a); break;
+    case QK_POW2: apply_kernel<QK_POW2><<<grid, block, 0, s>>>(a); break;
+    default: apply_kernel<QK_IDENT><<<grid, block, 0, s>>>(a); break;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fill(float *p, int64_t count, float value, cudaStream_t s)
+{
+    if (count <= 0) return cudaSuccess;
+    const int64_t want = (count + 255) / 256;
+    fill_kernel<<<static_cast<unsigned>(want < 152 * 64 ? want : 152 * 64), 256, 0, s>>>(p, count, value);
+    return cudaGetLastError();
+}
+
+}  // namespace ea

@@ -1,0 +1,219 @@
+"""GPU parity: the CUDA library, called through its C-ABI binding, against the oracle on the same
+seeded inputs, every round (see tests/parity.py for the tolerances)."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2205_14473_gb300 as ea
+from paper_2205_14473_gb300 import workloads as W
+
+from parity import Lockstep, expected_bits
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    yield
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def _run_host(cfg: ea.EAConfig, rounds: int, seed: int = 0, grad_scale: float = 1.0, x_scale: float = 1.0):
+    L = Lockstep(cfg)
+    rng = np.random.default_rng(seed)
+    x_host = (rng.standard_normal(cfg.d) * x_scale).astype(np.float32)
+    x_dev = torch.from_numpy(x_host.copy()).cuda()
+    for t in range(rounds):
+        scale = grad_scale * (10 ** rng.uniform(-1, 1))
+        gs = [(rng.standard_normal(cfg.d) * scale).astype(np.float32) for _ in range(cfg.n)]
+        L.round([torch.from_numpy(g).cuda() for g in gs], gs, x_dev, x_host)
+    assert L.gpu.bits_sent() == expected_bits(cfg, rounds)
+    return L
+
+
+# ----------------------------------------------------------------------- sizes and edge cases
+
+@pytest.mark.parametrize("d", [1, 3, 31, 32, 33, 4095, 4096, 4097, 12289, 20_000])
+@pytest.mark.parametrize("group", [4096, 0])
+def test_ragged_sizes(d, group):
+    cfg = ea.EAConfig(d=d, n=3, qw=W.sign_q(group), qs=W.sign_q(group), alpha=1e-3, seed=d)
+    _run_host(cfg, 3, seed=d)
+
+
+@pytest.mark.parametrize("n", [1, 2, 5])
+def test_worker_counts(n):
+    cfg = ea.EAConfig(d=9000, n=n, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-2)
+    _run_host(cfg, 4, seed=n)
+
+
+@pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
+@pytest.mark.parametrize("ef", [True, False])
+@pytest.mark.parametrize("group", [4096, 0, 1000])
+def test_placement_and_error_feedback(placement, ef, group):
+    cfg = ea.EAConfig(d=15_000, n=3, qw=W.sign_q(group), qs=W.sign_q(group), alpha=1e-3, placement=placement,
+                      error_feedback=ef, seed=11)
+    _run_host(cfg, 4, seed=3)
+
+
+_SEGS = (7, 1, 4096, 64, 5000, 3, 8192, 100, 11)
+
+
+@pytest.mark.parametrize("qw,qs,gs", [
+    (W.uniform_q(4, 4096, True), W.uniform_q(8, 4096, False), 1e-3),      # the c4 pair
+    (W.uniform_q(2, 0, False), W.uniform_q(2, 0, True), 1.0),             # Example 1 with k = 1
+    (W.uniform_q(16, 1000, True), W.uniform_q(16, 4096, False), 1.0),
+    (W.QuantSpec(W.Q_UNIFORM_MAX, 8, -1, _SEGS), W.sign_q(-1, _SEGS), 1.0),
+    (W.pow2_q(-17, -11, 4), W.pow2_q(-17, -11, 4), 1e-4),                 # Example 2, the paper's k, K
+    (W.pow2_q(-20, -5, 8), W.sign_q(4096), 1e-3),
+    (W.identity_q(), W.identity_q(), 1.0),                                # "Ours_full"
+    (W.sign_q(4096), W.uniform_q(4, 0, True), 1.0),
+    (W.identity_q(), W.sign_q(8192), 1.0),
+])
+@pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
+def test_quantizer_kinds(qw, qs, gs, placement):
+    d = sum(_SEGS)
+    cfg = ea.EAConfig(d=d, n=3, qw=qw, qs=qs, alpha=1e-3, placement=placement, seed=5)
+    _run_host(cfg, 4, seed=9, grad_scale=gs)
+
+
+def test_replicas_are_identical_and_protocol():
+    cfg = ea.EAConfig(d=10_000, n=2, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-3)
+    rnd = ea.EARound(cfg)
+    g = torch.randn(10_000, device="cuda")
+    x1 = torch.randn(10_000, device="cuda")
+    x2 = x1.clone()
+    with pytest.raises(ea.EAError) as ex:
+        rnd.apply(x1)
+    assert ex.value.status == ea.EA_E_ORDER
+    rnd.worker_compress(0, g)
+    with pytest.raises(ea.EAError) as ex:
+        rnd.worker_compress(0, g)
+    assert ex.value.status == ea.EA_E_ORDER
+    with pytest.raises(ea.EAError) as ex:
+        rnd.server_step()
+    assert ex.value.status == ea.EA_E_ORDER
+    gbuf = torch.empty(10_004, device="cuda")
+    with pytest.raises(ea.EAError) as ex:
+        ea.ea_worker_compress(rnd.h, 1, gbuf.data_ptr() + 4)
+    assert ex.value.status == ea.EA_E_ALIGN
+    with pytest.raises(ea.EAError):
+        rnd.worker_compress(2, g)
+    rnd.worker_compress(1, g)
+    rnd.server_step()
+    rnd.apply(x1)
+    rnd.apply(x2)
+    rnd.sync()
+    assert torch.equal(x1, x2)
+    assert rnd.t == 1
+
+
+# ------------------------------------------------------------------------- the five workloads
+
+def _dev_grads(w: W.Workload, t: int, bufs):
+    for i, b in enumerate(bufs):
+        W.gradient_device(w, i, t, b)
+    return bufs
+
+
+def test_c1_full():
+    w = W.WORKLOADS["c1"]
+    cfg = ea.EAConfig.from_workload(w)
+    L = Lockstep(cfg)
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(w.d, np.float32)
+    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    for t in range(w.rounds):
+        _dev_grads(w, t, bufs)
+        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (2_622_720, 2_622_720)
+
+
+def test_c2_quadratic_toy_full():
+    """The quadratic toy at d = 1e6, n = 8, all 1,000 rounds; both sides form g = (x - x*) + 0.1 xi
+    from their own x; ||x - x*|| decreases."""
+    w = W.WORKLOADS["c2"]
+    cfg = ea.EAConfig.from_workload(w)
+    L = Lockstep(cfg, threads=8)
+    xs_host = W.xstar_host(w)
+    xs_dev = torch.from_numpy(xs_host).cuda()
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(w.d, np.float32)
+    noise = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    dist = [float(np.linalg.norm(x_host - xs_host))]
+    for t in range(w.rounds):
+        _dev_grads(w, t, noise)
+        g_dev = [W.quadratic_gradient(x_dev, xs_dev, nz) for nz in noise]
+        g_host = [W.quadratic_gradient(x_host, xs_host, L.host(nz)) for nz in noise]
+        L.round(g_dev, g_host, x_dev, x_host)
+        if (t + 1) % 50 == 0:
+            dist.append(float(torch.linalg.vector_norm(x_dev - xs_dev)))
+    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (8_000_256_000, 8_000_256_000)
+    assert dist[-1] < 0.1 * dist[0]
+    assert all(b < a for a, b in zip(dist[:6], dist[1:7]))
+
+
+def test_c3_resnet18_all_tensors_first_rounds():
+    w = W.WORKLOADS["c3"]
+    cfg = ea.EAConfig.from_workload(w)
+    L = Lockstep(cfg, threads=16)
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(w.d, np.float32)
+    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    for t in range(3):
+        _dev_grads(w, t, bufs)
+        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+
+
+def test_c3_resnet18_sampled_tensors_all_rounds():
+    """All 100 rounds at full size; the oracle follows 14 of the 62 tensors (per-tensor scales make
+    the round separable by tensor), including the smallest, the largest and fc."""
+    w = W.WORKLOADS["c3"]
+    cfg = ea.EAConfig.from_workload(w)
+    groups = [0, 1, 2, 3, 8, 16, 25, 33, 41, 47, 52, 56, 60, 61]
+    L = Lockstep(cfg, sample_groups=groups, threads=16)
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(L.d_o, np.float32)
+    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    for t in range(w.rounds):
+        _dev_grads(w, t, bufs)
+        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (18_706_393_600, 18_706_393_600)
+
+
+@pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
+def test_c4_sampled_blocks_all_rounds(placement):
+    w = W.WORKLOADS["c4"]
+    cfg = ea.EAConfig.from_workload(w, placement=placement)
+    L = Lockstep(cfg, sample_groups=W.sample_blocks(w, 48), threads=8)
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(L.d_o, np.float32)
+    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    for t in range(w.rounds):
+        _dev_grads(w, t, bufs)
+        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (176_343_756_800, 352_343_756_800)
+    del L, bufs, x_dev
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
+def test_c5_sampled_blocks_all_rounds(placement):
+    """d = 1.558e9, n = 8 on one GPU (W: ~213 GB resident, S: ~126 GB), all 10 rounds; the oracle
+    follows 32 of the 380,372 blocks, including the first and the ragged last one."""
+    w = W.WORKLOADS["c5"]
+    cfg = ea.EAConfig.from_workload(w, placement=placement)
+    L = Lockstep(cfg, sample_groups=W.sample_blocks(w, 32), threads=8)
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(L.d_o, np.float32)
+    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    for t in range(w.rounds):
+        _dev_grads(w, t, bufs)
+        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (125_613_752_320, 125_613_752_320)
+    del L, bufs, x_dev
+    torch.cuda.empty_cache()
