@@ -41,10 +41,14 @@ def _peaks():
         return 6800.0, "fallback"
 
 
+_OVERRIDE = {}
+
+
 def _workload(name: str):
     from paper_2205_14473_gb300 import workloads as W
 
-    return W.WORKLOADS[name]
+    w = W.WORKLOADS[name]
+    return w.with_(**_OVERRIDE) if _OVERRIDE else w
 
 
 def _describe(w, placement: int) -> str:
@@ -400,8 +404,14 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--d", type=int, default=None, help="override d (small profiling cases)")
+    ap.add_argument("--n", type=int, default=None, help="override the worker count")
     args = ap.parse_args()
 
+    if args.d:
+        _OVERRIDE["d"] = args.d
+    if args.n:
+        _OVERRIDE["n"] = args.n
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -19,6 +19,7 @@ namespace {
 thread_local std::string g_last_error;  // failures that have no handle yet
 
 constexpr size_t kAlign = 256;
+constexpr uint32_t kStatusTimeoutBit = 1u;  // set by kernels whose bounded waits gave up
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -38,7 +39,7 @@ struct QHost {
 // Sizes of every workspace buffer, in the order they are carved.
 struct Layout {
     size_t e_w, m_w, v_w, e_s, m_s, v_s, codes_w, scales_w, codes_s, scales_s, partials;
-    size_t off_w, tg_w, pb_w, off_s, tg_s, pb_s;
+    size_t off_w, tg_w, pb_w, off_s, tg_s, pb_s, status;
     int64_t dpad, wcode_stride, wscale_stride;
 };
 
@@ -54,6 +55,8 @@ struct ea_handle {
     uint32_t *wcodes = nullptr, *scodes = nullptr;
     float *wscales = nullptr, *sscales = nullptr;
     double *partials = nullptr;
+    uint32_t *status = nullptr;
+    StagePlan splan{};
     Hyper hp{};
     int64_t t = 0;
     std::vector<unsigned char> compressed;
@@ -232,13 +235,14 @@ Layout make_layout(const ea_config &c, const QHost &qw, const QHost &qs)
     L.off_s = qs.gkind == GK_SEG ? qs.offsets.size() * 8 : 0;
     L.tg_s = qs.gkind == GK_SEG ? static_cast<size_t>(n_tiles) * 4 : 0;
     L.pb_s = qs.pass == PASS_STASH ? qs.pair_base.size() * 8 : 0;
+    L.status = 4;
     return L;
 }
 
 size_t layout_bytes(const Layout &L)
 {
     const size_t parts[] = {L.e_w, L.m_w, L.v_w, L.e_s, L.m_s, L.v_s, L.codes_w, L.scales_w, L.codes_s,
-                            L.scales_s, L.partials, L.off_w, L.tg_w, L.pb_w, L.off_s, L.tg_s, L.pb_s};
+                            L.scales_s, L.partials, L.off_w, L.tg_w, L.pb_w, L.off_s, L.tg_s, L.pb_s, L.status};
     size_t total = 0;
     for (size_t p : parts) total += align_up(p, kAlign);
     return total;
@@ -273,6 +277,46 @@ uint64_t message_bits(const QHost &q, int64_t d)
 {
     return static_cast<uint64_t>(d) * static_cast<uint64_t>(q.bits) +
            (q.has_scales ? 32ull * static_cast<uint64_t>(q.n_groups) : 0ull);
+}
+
+// Shared-memory staging of the server's inputs (see server_staged_kernel): one stage holds a
+// tile's e_s (+ m_s, v_s) and the n workers' code chunks and scales.  Enabled when both messages
+// have one scale per 4096-tile (or none) and a stage fits the budget: 100 KB per CTA and two CTAs
+// per SM with Adam at the workers; 200 KB and one CTA per SM (more registers) with Adam at the
+// server, whose stages are larger.
+StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs, int64_t n_tiles, int sms)
+{
+    StagePlan P{};
+    const bool qs_ok = !qs.has_scales || qs.pass == PASS_FUSED;
+    const bool qw_ok = !qw.has_scales || qw.pass == PASS_FUSED;
+    if (!qs_ok || !qw_ok || sms <= 0) return P;
+    const bool server_adam = c.placement == EA_ADAM_AT_SERVER;
+    uint32_t off = 0;
+    P.off_a = off;
+    off += 4 * kTile;
+    if (server_adam) {
+        P.off_b = off;
+        off += 4 * kTile;
+        P.off_c = off;
+        off += 4 * kTile;
+    }
+    const uint32_t budget = server_adam ? 200 * 1024 : 100 * 1024;
+    P.code_chunk = static_cast<uint32_t>(kTile / 8 * qw.bits);
+    P.off_codes = off;
+    const uint64_t codes = static_cast<uint64_t>(P.code_chunk) * c.n;
+    if (codes > budget / 2) return P;
+    off += static_cast<uint32_t>(codes);
+    P.off_scales = off;
+    off += static_cast<uint32_t>(align_up(4 * static_cast<size_t>(c.n), 16));
+    P.stage_bytes = static_cast<uint32_t>(align_up(off, 128));
+    if (2 * P.stage_bytes > budget) return P;
+    P.stages = std::max(2, std::min(6, static_cast<int>(budget / P.stage_bytes)));
+    const uint32_t bars = static_cast<uint32_t>(align_up(2 * 8 * static_cast<size_t>(P.stages), 128));
+    P.smem_bytes = bars + static_cast<uint32_t>(P.stages) * P.stage_bytes;
+    const int per_sm = (!server_adam && 2 * (P.smem_bytes + 4096) <= 228 * 1024) ? 2 : 1;
+    P.grid = static_cast<int>(std::min<int64_t>(n_tiles, static_cast<int64_t>(sms) * per_sm));
+    P.enabled = 1;
+    return P;
 }
 
 int check_dev_ptr(ea_handle *h, const void *p, const char *what)
@@ -375,6 +419,11 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->qs.d_offsets = reinterpret_cast<int64_t *>(take(L.off_s));
     h->qs.d_tile_group = reinterpret_cast<int32_t *>(take(L.tg_s));
     h->qs.d_pair_base = reinterpret_cast<int64_t *>(take(L.pb_s));
+    h->status = reinterpret_cast<uint32_t *>(take(L.status));
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+        h->splan = make_server_plan(*cfg, h->qw, h->qs, h->n_tiles, sms);
 
     // Algorithm 2: m_0 = 0, v_0 = eps, e_1 = 0; Algorithm 1: e_1 = 0.  Messages start zeroed.
     cudaStream_t s = h->stream;
@@ -463,6 +512,10 @@ int ea_server_step(ea_handle *h)
     a.seed = h->cfg.seed;
     a.t = static_cast<uint32_t>(h->t);
     a.partials = h->partials;
+    a.dpad = h->lay.dpad;
+    a.wcode_bytes = h->lay.wcode_stride * 4;
+    a.status = h->status;
+    a.plan = h->splan;
     const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
     int r = check_cuda(h, W ? launch_server_w(a, h->stream) : launch_server_s(a, h->stream), "server launch");
     if (r == EA_OK && h->qs.pass == PASS_STASH)
@@ -545,7 +598,18 @@ int ea_sync_status(ea_handle *h)
     if (!h) return fail(nullptr, EA_E_INVAL, "handle is NULL");
     int r = check_cuda(h, cudaStreamSynchronize(h->stream), "stream synchronize");
     if (r != EA_OK) return r;
-    return check_cuda(h, cudaGetLastError(), "pending error");
+    r = check_cuda(h, cudaGetLastError(), "pending error");
+    if (r != EA_OK) return r;
+    uint32_t st = 0;
+    r = check_cuda(h, cudaMemcpy(&st, h->status, sizeof st, cudaMemcpyDeviceToHost), "status read");
+    if (r != EA_OK) return r;
+    if (st) {
+        cudaMemset(h->status, 0, sizeof st);
+        if (st & kStatusTimeoutBit)
+            return fail(h, EA_E_TIMEOUT, "a device-side wait exceeded its time limit (status 0x%x)", st);
+        return fail(h, EA_E_DEVICE_CHECK, "device status 0x%x", st);
+    }
+    return EA_OK;
 }
 
 const char *ea_last_error(const ea_handle *h)

@@ -77,6 +77,10 @@ __device__ __forceinline__ void df_accumulate(DF &acc, float x)
     acc.lo = __fadd_rn(acc.lo, e);
 }
 
+// Barrier over the 256 compute threads (named barrier 1), so that a CTA may also hold a producer
+// warp that does not take part in the reductions.
+__device__ __forceinline__ void compute_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kThreads) : "memory"); }
+
 // CTA-wide sum; every thread receives the same binary64 value (fixed combination order).
 __device__ __forceinline__ double block_sum(DF v, DF *red, double *bcast)
 {
@@ -87,15 +91,56 @@ __device__ __forceinline__ double block_sum(DF v, DF *red, double *bcast)
     }
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if (lane == 0) red[warp] = v;
-    __syncthreads();
+    compute_sync();
     if (threadIdx.x == 0) {
         DF t = red[0];
 #pragma unroll
         for (int w = 1; w < kWarps; ++w) t = df_add(t, red[w]);
         *bcast = static_cast<double>(t.hi) + static_cast<double>(t.lo);
     }
-    __syncthreads();
-    return *bcast;
+    compute_sync();
+    const double r = *bcast;
+    return r;
+}
+
+// Group scale of the scaled sign, ||u||_1 / G, for a group that is exactly this CTA's tile.  One
+// barrier: every thread combines the eight warp totals in the same order, so all get the same
+// value without a broadcast.  For G a power of two, RN32((hi + lo) / G) = RN32(hi + lo) * 2^-k is
+// one binary32 addition and an exact scaling; other lengths (a ragged last tile) divide in
+// binary64.  The caller must barrier before `red` is reused.
+__device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        DF w{__shfl_down_sync(0xffffffffu, v.hi, o), __shfl_down_sync(0xffffffffu, v.lo, o)};
+        v = df_add(v, w);
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) red[warp] = v;
+    compute_sync();
+    DF t = red[0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) t = df_add(t, red[w]);
+    if (len <= 0) return 0.0f;
+    if ((len & (len - 1)) == 0) {  // len <= 4096 here: the factor 2^-k is a normal binary32
+        const int k = __ffsll(static_cast<long long>(len)) - 1;
+        return __fmul_rn(__fadd_rn(t.hi, t.lo), __uint_as_float(static_cast<uint32_t>(127 - k) << 23));
+    }
+    const double l1 = static_cast<double>(t.hi) + static_cast<double>(t.lo);
+    return __double2float_rn(__ddiv_rn(l1, static_cast<double>(len)));
+}
+
+// CTA-wide maximum for a group that is exactly this CTA's tile: one barrier, every thread combines
+// the warp maxima itself.  The caller must barrier before `red` is reused.
+__device__ __forceinline__ float block_max_all(float a, uint32_t *red)
+{
+    const uint32_t b = __reduce_max_sync(0xffffffffu, __float_as_uint(a));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = b;
+    compute_sync();
+    uint32_t m = red[0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) m = max(m, red[w]);
+    return __uint_as_float(m);
 }
 
 // CTA-wide maximum of non-negative values (exact: compares bit patterns).
@@ -104,15 +149,16 @@ __device__ __forceinline__ float block_max(float a, uint32_t *red, float *bcast)
     const uint32_t b = __reduce_max_sync(0xffffffffu, __float_as_uint(a));
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if (lane == 0) red[warp] = b;
-    __syncthreads();
+    compute_sync();
     if (threadIdx.x == 0) {
         uint32_t m = red[0];
 #pragma unroll
         for (int w = 1; w < kWarps; ++w) m = max(m, red[w]);
         *bcast = __uint_as_float(m);
     }
-    __syncthreads();
-    return *bcast;
+    compute_sync();
+    const float r = *bcast;
+    return r;
 }
 
 // Group scale of the scaled sign: ||u||_1 / G, the division in binary64, one rounding to binary32.
@@ -210,6 +256,13 @@ __device__ __forceinline__ constexpr bool has_scale()
     return QK == QK_SIGN || QK == QK_UNIF;
 }
 
+// Code width: fixed by the kind for the sign (1) and identity (32) mappings, else configured.
+template <int QK>
+__device__ __forceinline__ int code_bits(const QParams &q)
+{
+    return QK == QK_SIGN ? 1 : (QK == QK_IDENT ? 32 : q.bits);
+}
+
 // ----------------------------------------------------------------------------- scale groups
 
 __device__ __forceinline__ int64_t group_begin(const Grouping &g, int64_t gi, int64_t d)
@@ -285,6 +338,7 @@ __device__ __forceinline__ uint32_t spread8_by4(uint32_t x)
 // called by all 32 lanes of the warp.  Codes of coordinates >= d are 0 (caller's job).
 // b = 1: one ballot per component; lanes 8g .. 8g+7 fill word (q_lane0 / 8) + g, whose bit
 // 4l + c is component c of lane 8g + l.
+template <bool FULL = false>
 __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64_t q, int bits, const uint32_t c[4],
                                              int64_t n_words)
 {
@@ -299,7 +353,7 @@ __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64
             const uint32_t w = spread8_by4(b0 >> sh) | (spread8_by4(b1 >> sh) << 1) | (spread8_by4(b2 >> sh) << 2) |
                                (spread8_by4(b3 >> sh) << 3);
             const int64_t wi = ((q - lane) >> 3) + lane;  // q - lane is lane 0's slot
-            if (wi < n_words) words[wi] = w;
+            if (FULL || wi < n_words) words[wi] = w;
         }
     } else if (bits <= 8) {
         uint32_t v = 0;
@@ -311,12 +365,12 @@ __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64
         if (per_word >= 2) v |= __shfl_xor_sync(0xffffffffu, v, 1);
         if (per_word >= 4) v |= __shfl_xor_sync(0xffffffffu, v, 2);
         const int64_t wi = (q * bits) >> 3;
-        if (pos == 0 && wi < n_words) words[wi] = v;
+        if (pos == 0 && (FULL || wi < n_words)) words[wi] = v;
     } else if (bits == 16) {
-        if (2 * q < n_words)
+        if (FULL || 2 * q < n_words)
             reinterpret_cast<uint2 *>(words)[q] = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
     } else {
-        if (4 * q < n_words) reinterpret_cast<uint4 *>(words)[q] = make_uint4(c[0], c[1], c[2], c[3]);
+        if (FULL || 4 * q < n_words) reinterpret_cast<uint4 *>(words)[q] = make_uint4(c[0], c[1], c[2], c[3]);
     }
 }
 
@@ -340,11 +394,13 @@ __device__ __forceinline__ void to_arr(const float4 &v, float a[4])
 
 __device__ __forceinline__ float4 to_f4(const float a[4]) { return make_float4(a[0], a[1], a[2], a[3]); }
 
-// Load slot q of p (4 coordinates from 4q) into a; coordinates >= d read as 0.
+// Load slot q of p (4 coordinates from 4q) into a; coordinates >= d read as 0.  FULL: the caller
+// knows the slot lies inside [0, d).
+template <bool FULL = false>
 __device__ __forceinline__ void load4(const float *__restrict__ p, int64_t q, int64_t d, float a[4])
 {
     const int64_t j0 = 4 * q;
-    if (j0 + 4 <= d) {
+    if (FULL || j0 + 4 <= d) {
         to_arr(__ldcs(reinterpret_cast<const float4 *>(p) + q), a);
     } else {
 #pragma unroll
@@ -352,10 +408,11 @@ __device__ __forceinline__ void load4(const float *__restrict__ p, int64_t q, in
     }
 }
 
+template <bool FULL = false>
 __device__ __forceinline__ void store4(float *__restrict__ p, int64_t q, int64_t d, const float a[4])
 {
     const int64_t j0 = 4 * q;
-    if (j0 + 4 <= d) {
+    if (FULL || j0 + 4 <= d) {
         __stcs(reinterpret_cast<float4 *>(p) + q, to_f4(a));
     } else {
 #pragma unroll

@@ -59,6 +59,20 @@ struct WorkerArgs {
     double *partials;
 };
 
+// Shared-memory staging plan of the pipelined (persistent, bulk-copy) kernels.  A stage holds one
+// tile's inputs; byte offsets are relative to the stage start and 128-byte aligned.
+struct StagePlan {
+    int enabled;               // 0: use the direct-load kernel
+    int stages;                // pipeline depth
+    int grid;                  // persistent CTAs
+    uint32_t stage_bytes;      // bytes of one stage
+    uint32_t smem_bytes;       // dynamic shared memory per CTA (barriers + stages)
+    uint32_t off_a, off_b, off_c, off_d;  // up to four 16 KB state tiles (kernel-specific meaning)
+    uint32_t off_codes;        // n code chunks of code_chunk bytes
+    uint32_t code_chunk;       // bytes of one worker's codes for one tile (4096 b / 8)
+    uint32_t off_scales;       // n worker scales (binary32)
+};
+
 struct ServerArgs {
     int64_t d, n_tiles;
     int n;
@@ -75,6 +89,10 @@ struct ServerArgs {
     uint64_t seed;
     uint32_t t;
     double *partials;
+    int64_t dpad;             // padded length of e_s, m_s, v_s (multiple of 64)
+    int64_t wcode_bytes;      // padded bytes of one worker's code stream (multiple of 256)
+    uint32_t *status;         // device status word (timeouts)
+    StagePlan plan;
 };
 
 // Second pass of PASS_STASH: encode the stashed input in buf, leave the residual in buf.

@@ -1,6 +1,7 @@
 // ea_server.cuh -- the server's round (Algorithm 1) on one 4096-coordinate tile.
 #pragma once
 
+#include "ea_async.cuh"
 #include "ea_tile.cuh"
 
 namespace ea {
@@ -74,6 +75,8 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
     }
 
     const float nf = static_cast<float>(a.n);
+    const bool pow2n = (a.n & (a.n - 1)) == 0;
+    const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
     float u[kSlots][4];
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
@@ -81,7 +84,7 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
         const int64_t j0 = 4 * q;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            float step = __fdiv_rn(acc[k][i], nf);
+            float step = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
             if (MODE == MODE_S) step = adam_step(step, ms[k][i], vs[k][i], a.hp);
             u[k][i] = (j0 + i < d) ? __fadd_rn(step, es[k][i]) : 0.0f;
         }
@@ -94,9 +97,225 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
                     static_cast<uint32_t>(a.n), a.t, a.partials, sm);
 }
 
+
+// Load the four codes of local slot ls (0 .. 1023) of a tile's code chunk held in shared memory.
+__device__ __forceinline__ void load_codes4_smem(const uint32_t *words, int ls, int bits, uint32_t c[4])
+{
+    if (bits <= 8) {
+        const uint32_t w = words[(ls * bits) >> 3];
+        const int sh = ((ls * bits) & 7) * 4;
+        const uint32_t mask = (1u << bits) - 1u;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) c[i] = (w >> (sh + i * bits)) & mask;
+    } else if (bits == 16) {
+        const uint2 w = reinterpret_cast<const uint2 *>(words)[ls];
+        c[0] = w.x & 0xffffu;
+        c[1] = w.x >> 16;
+        c[2] = w.y & 0xffffu;
+        c[3] = w.y >> 16;
+    } else {
+        const uint4 w = reinterpret_cast<const uint4 *>(words)[ls];
+        c[0] = w.x;
+        c[1] = w.y;
+        c[2] = w.z;
+        c[3] = w.w;
+    }
+}
+
+// All 256 compute threads agree on `ok` (named barrier 1 with an AND reduction).
+__device__ __forceinline__ bool compute_all(bool ok)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.and.pred q, 1, %2, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(ok ? 1u : 0u), "n"(kThreads)
+        : "memory");
+    return r != 0;
+}
+
+// One tile of the staged server on the compute warps: the stage `st` holds e_s (m_s, v_s), the
+// workers' code chunks and scales.  The stage is released (arrive on `empty`) as soon as it has
+// been read, before the re-quantization.
+template <int MODE, int QW, int QS, bool FULL>
+__device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
+                                                   uint64_t *empty, int Lw, float Lwf, const float *utab,
+                                                   TileSmem &sm)
+{
+    const StagePlan &P = a.plan;
+    const int64_t d = a.d;
+    const int bw = code_bits<QW>(a.qw);
+    const float nf = static_cast<float>(a.n);
+    const bool pow2n = (a.n & (a.n - 1)) == 0;
+    const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
+    float acc[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+    const float *sc = reinterpret_cast<const float *>(st + P.off_scales);
+#pragma unroll 4
+    for (int w = 0; w < a.n; ++w) {
+        const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
+        const float sw = has_scale<QW>() ? sc[w] : 0.0f;
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            uint32_t c[4];
+            load_codes4_smem(cw, k * kThreads + threadIdx.x, bw, c);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
+        }
+    }
+    // e_s (and m_s, v_s) are read from the stage only now, to keep registers for the sums
+    float u[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int ls = k * kThreads + threadIdx.x;
+        const int64_t q = slot_of(tile, k);
+        const int64_t j0 = 4 * q;
+        float es[4], ms[4], vs[4];
+        to_arr(reinterpret_cast<const float4 *>(st + P.off_a)[ls], es);
+        if (MODE == MODE_S) {
+            to_arr(reinterpret_cast<const float4 *>(st + P.off_b)[ls], ms);
+            to_arr(reinterpret_cast<const float4 *>(st + P.off_c)[ls], vs);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float step = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
+            if (MODE == MODE_S) step = adam_step(step, ms[i], vs[i], a.hp);
+            u[k][i] = (FULL || j0 + i < d) ? __fadd_rn(step, es[i]) : 0.0f;
+        }
+        if (MODE == MODE_S && (FULL || j0 < d)) {
+            store4<FULL>(a.ms, q, d, ms);
+            store4<FULL>(a.vs, q, d, vs);
+        }
+    }
+    // the stage is no longer read: hand it back to the producer before the tile's epilogue
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(empty);
+    finish_tile<QS, FULL>(u, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.pass, a.seed,
+                          static_cast<uint32_t>(a.n), a.t, a.partials, sm);
+}
+
+// The server's round with its inputs staged through shared memory.  Persistent CTAs of 8 compute
+// warps and 1 producer warp: the producer streams, for each of the CTA's tiles, the e_s tile (and
+// m_s, v_s with Adam at the server) and the n workers' code chunks with bulk copies, and the n
+// worker scales with 4-byte cp.async, into a ring of stages guarded by full/empty mbarriers; the
+// compute warps decode, average, re-quantize and write e_s and the broadcast straight to HBM.
+// Used when Q_s scales are per 4096-tile (or absent) and Q_w's are per 4096-tile (or absent).
+template <int MODE, int QW, int QS>
+__global__ void __launch_bounds__(kThreads + 32, MODE == MODE_W ? 2 : 1) server_staged_kernel(const ServerArgs a)
+{
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ TileSmem sm;
+    __shared__ float utab[256];
+    const StagePlan &P = a.plan;
+    const int S = P.stages;
+    uint64_t *full = reinterpret_cast<uint64_t *>(dsm);
+    uint64_t *empty = full + S;
+    unsigned char *stage0 = dsm + 128 * ((2 * S * 8 + 127) / 128);
+    constexpr bool scaled_w = has_scale<QW>();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1 + (scaled_w ? 32 : 0));
+            mbar_init(&empty[s], kWarps);
+        }
+        mbar_init_fence();
+    }
+    const int Lw = (QW == QK_UNIF) ? unif_L(a.qw.bits) : 0;
+    const float Lwf = static_cast<float>(Lw);
+    const bool use_tab = QW == QK_UNIF && a.qw.bits <= 8;
+    if (use_tab)
+        for (int i = threadIdx.x; i <= 2 * Lw; i += blockDim.x) utab[i] = __fdiv_rn(static_cast<float>(i - Lw), Lwf);
+    __syncthreads();
+
+    if (warp == kWarps) {  // ---------------------------------------------------------- producer
+        int64_t it = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
+            const int s = static_cast<int>(it % S);
+            if (it >= S && !mbar_wait(&empty[s], static_cast<uint32_t>(((it / S) & 1) ^ 1))) {
+                ok = false;
+                break;
+            }
+            unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
+            const int64_t lo = tile * kTile;
+            const uint32_t vb = static_cast<uint32_t>(min(static_cast<int64_t>(kTile), a.dpad - lo) * 4);
+            const int64_t coff = tile * static_cast<int64_t>(P.code_chunk);
+            const uint32_t cb = static_cast<uint32_t>(min(static_cast<int64_t>(P.code_chunk), a.wcode_bytes - coff));
+            if (lane == 0) {
+                mbar_arrive_expect_tx(&full[s], vb * (MODE == MODE_S ? 3u : 1u) + cb * static_cast<uint32_t>(a.n));
+                bulk_g2s(st + P.off_a, a.es + lo, vb, &full[s]);
+                if (MODE == MODE_S) {
+                    bulk_g2s(st + P.off_b, a.ms + lo, vb, &full[s]);
+                    bulk_g2s(st + P.off_c, a.vs + lo, vb, &full[s]);
+                }
+                const unsigned char *wb = reinterpret_cast<const unsigned char *>(a.wwords) + coff;
+                for (int w = 0; w < a.n; ++w)
+                    bulk_g2s(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk, wb + w * a.wcode_bytes, cb,
+                             &full[s]);
+            }
+            if (scaled_w) {
+                float *sc = reinterpret_cast<float *>(st + P.off_scales);
+                for (int w = lane; w < a.n; w += 32) cp_async4(sc + w, a.wscales + w * a.wscales_stride + tile);
+                cp_async_arrive_noinc(&full[s]);
+            }
+        }
+        // the copies of the last stages must land before the CTA may exit
+        for (int64_t j = (it > S ? it - S : 0); j < it; ++j)
+            if (!mbar_wait(&full[j % S], static_cast<uint32_t>((j / S) & 1))) ok = false;
+        if (!ok && lane == 0) report_status(a.status, kStatusTimeout);
+        return;
+    }
+
+    // ------------------------------------------------------------------------- compute warps
+    const int64_t d = a.d;
+    int64_t it = 0;
+    for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
+        const int s = static_cast<int>(it % S);
+        const bool ok = compute_all(mbar_wait(&full[s], static_cast<uint32_t>((it / S) & 1)));
+        if (!ok) {
+            if (threadIdx.x == 0) report_status(a.status, kStatusTimeout);
+            break;
+        }
+        const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
+        if ((tile + 1) * kTile <= d)
+            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, sm);
+        else
+            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, sm);
+    }
+}
+
+template <int MODE, int QW, int QS>
+static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
+{
+    static bool attr_set = false;
+    if (!attr_set) {
+        const cudaError_t e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>,
+                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    server_staged_kernel<MODE, QW, QS><<<a.plan.grid, kThreads + 32, a.plan.smem_bytes, s>>>(a);
+    return cudaGetLastError();
+}
+
 template <int MODE, int QW>
 static cudaError_t launch_server_qw(const ServerArgs &a, cudaStream_t s)
 {
+    if (a.plan.enabled) {
+        switch (a.qs.kind) {
+        case QK_SIGN: return launch_server_staged<MODE, QW, QK_SIGN>(a, s);
+        case QK_UNIF: return launch_server_staged<MODE, QW, QK_UNIF>(a, s);
+        case QK_POW2: return launch_server_staged<MODE, QW, QK_POW2>(a, s);
+        default: return launch_server_staged<MODE, QW, QK_IDENT>(a, s);
+        }
+    }
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
     switch (a.qs.kind) {
     case QK_SIGN: server_kernel<MODE, QW, QK_SIGN><<<grid, block, 0, s>>>(a); break;

@@ -22,44 +22,46 @@ __device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
 }
 
 // Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
-template <int QK>
+// FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
+template <int QK, bool FULL>
 __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
                                              const QParams &q, uint32_t *words, float *resid, int ef,
                                              uint64_t seed, uint32_t id, uint32_t t)
 {
-    const int L = (QK == QK_UNIF) ? unif_L(q.bits) : 0;
+    const int bits = code_bits<QK>(q);
+    const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
     const float Lf = static_cast<float>(L);
-    const int64_t n_words = (d * q.bits + 31) >> 5;
+    const int64_t n_words = (d * bits + 31) >> 5;
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t qs = slot_of(tile, k);
         const int64_t j0 = 4 * qs;
         float U[4] = {0.f, 0.f, 0.f, 0.f};
-        if (QK == QK_UNIF && q.stochastic && j0 < d) uniforms4(seed, id, t, j0, U);
+        if (QK == QK_UNIF && q.stochastic && (FULL || j0 < d)) uniforms4(seed, id, t, j0, U);
         uint32_t c[4];
         float e[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             float dec = 0.0f;
-            c[i] = (j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec) : 0u;
+            c[i] = (FULL || j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec) : 0u;
             e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;
         }
-        store_codes4(words, qs, q.bits, c, n_words);
-        if (ef && j0 < d) store4(resid, qs, d, e);
+        store_codes4<FULL>(words, qs, bits, c, n_words);
+        if (ef && (FULL || j0 < d)) store4<FULL>(resid, qs, d, e);
     }
 }
 
 // The tile's end for a quantizer with scale groups.
 //   PASS_FUSED: the tile is exactly one scale group (blocks of 4096): reduce, encode, store.
 //   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
-template <int QK>
+template <int QK, bool FULL = false>
 __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile, int64_t d, const QParams &q,
                                             uint32_t *words, float *scales, float *resid, int ef, int pass,
                                             uint64_t seed, uint32_t id, uint32_t t, double *partials,
                                             TileSmem &sm)
 {
     if constexpr (!has_scale<QK>()) {
-        encode_store<QK>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t);
+        encode_store<QK, FULL>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t);
         return;
     } else {
         const int64_t tile_lo = tile * kTile;
@@ -72,24 +74,24 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
                 for (int k = 0; k < kSlots; ++k)
 #pragma unroll
                     for (int i = 0; i < 4; ++i) df_accumulate(acc, fabsf(u[k][i]));  // invalid u are 0
-                s = sign_scale(block_sum(acc, sm.red, &sm.bcast), tile_hi - tile_lo);
+                s = block_sign_scale(acc, tile_hi - tile_lo, sm.red);
             } else {
                 float mx = 0.0f;
 #pragma unroll
                 for (int k = 0; k < kSlots; ++k)
 #pragma unroll
                     for (int i = 0; i < 4; ++i) mx = fmaxf(mx, fabsf(u[k][i]));
-                s = block_max(mx, sm.redm, &sm.bcastf);
+                s = block_max_all(mx, sm.redm);
             }
             if (threadIdx.x == 0) scales[tile] = s;
-            encode_store<QK>(u, s, tile, d, q, words, resid, ef, seed, id, t);
+            encode_store<QK, FULL>(u, s, tile, d, q, words, resid, ef, seed, id, t);
             return;
         }
         // PASS_STASH
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
             const int64_t qs = slot_of(tile, k);
-            if (4 * qs < d) store4(resid, qs, d, u[k]);
+            if (FULL || 4 * qs < d) store4<FULL>(resid, qs, d, u[k]);
         }
         const Grouping &G = q.grp;
         for (int64_t gi = first_group_of_tile(G, tile);; ++gi) {

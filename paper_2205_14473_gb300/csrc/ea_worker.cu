@@ -3,26 +3,20 @@
 
 namespace ea {
 
-// Algorithm 2 for one worker on one 4096-coordinate tile.  With Adam at the worker:
-//   v <- beta2 v + (1-beta2) g^2, m <- beta1 m + (1-beta1) g, u = alpha m / sqrt(v) + e;
-// with Adam at the server: u = g + e.  Then Q_w(u) and e <- u - Q_w(u) (finish_tile).
-// HBM traffic per coordinate: 16 B read + 12 B written + b/8 B of code (Adam at the worker).
-template <int MODE, int QK>
-__global__ void __launch_bounds__(kThreads, 2) worker_kernel(const WorkerArgs a)
+// One tile of worker_kernel; FULL: the tile lies inside [0, d) (every tile but a ragged last one).
+template <int MODE, int QK, bool FULL>
+__device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, TileSmem &sm)
 {
-    __shared__ TileSmem sm;
-    const int64_t tile = blockIdx.x;
     const int64_t d = a.d;
-
     float g[kSlots][4], e[kSlots][4], m[kSlots][4], v[kSlots][4];
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t q = slot_of(tile, k);
-        load4(a.g, q, d, g[k]);
-        load4(a.e, q, d, e[k]);
+        load4<FULL>(a.g, q, d, g[k]);
+        load4<FULL>(a.e, q, d, e[k]);
         if (MODE == MODE_W) {
-            load4(a.m, q, d, m[k]);
-            load4(a.v, q, d, v[k]);
+            load4<FULL>(a.m, q, d, m[k]);
+            load4<FULL>(a.v, q, d, v[k]);
         }
     }
     float u[kSlots][4];
@@ -34,14 +28,27 @@ __global__ void __launch_bounds__(kThreads, 2) worker_kernel(const WorkerArgs a)
         for (int i = 0; i < 4; ++i) {
             float step = g[k][i];
             if (MODE == MODE_W) step = adam_step(g[k][i], m[k][i], v[k][i], a.hp);
-            u[k][i] = (j0 + i < d) ? __fadd_rn(step, e[k][i]) : 0.0f;
+            u[k][i] = (FULL || j0 + i < d) ? __fadd_rn(step, e[k][i]) : 0.0f;
         }
-        if (MODE == MODE_W && j0 < d) {
-            store4(a.m, q, d, m[k]);
-            store4(a.v, q, d, v[k]);
+        if (MODE == MODE_W && (FULL || j0 < d)) {
+            store4<FULL>(a.m, q, d, m[k]);
+            store4<FULL>(a.v, q, d, v[k]);
         }
     }
-    finish_tile<QK>(u, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t, a.partials, sm);
+    finish_tile<QK, FULL>(u, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t, a.partials, sm);
+}
+
+// Algorithm 2 for one worker on one 4096-coordinate tile.  With Adam at the worker:
+//   v <- beta2 v + (1-beta2) g^2, m <- beta1 m + (1-beta1) g, u = alpha m / sqrt(v) + e;
+// with Adam at the server: u = g + e.  Then Q_w(u) and e <- u - Q_w(u) (finish_tile).
+// HBM traffic per coordinate: 16 B read + 12 B written + b/8 B of code (Adam at the worker).
+template <int MODE, int QK>
+__global__ void __launch_bounds__(kThreads, 2) worker_kernel(const WorkerArgs a)
+{
+    __shared__ TileSmem sm;
+    const int64_t tile = blockIdx.x;
+    if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK, true>(a, tile, sm);
+    else worker_tile<MODE, QK, false>(a, tile, sm);
 }
 
 // Second pass, one CTA per scale group: combine the group's per-tile partial norms in a fixed
