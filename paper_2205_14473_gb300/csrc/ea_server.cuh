@@ -98,6 +98,16 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
 }
 
 
+// Bits 0, 4, ..., 28 of x moved to bits 0 .. 7 (the inverse of spread8_by4).
+__device__ __forceinline__ uint32_t gather_every4(uint32_t x)
+{
+    x &= 0x11111111u;
+    x = (x | (x >> 3)) & 0x03030303u;
+    x = (x | (x >> 6)) & 0x000f000fu;
+    x = (x | (x >> 12)) & 0x000000ffu;
+    return x;
+}
+
 // Load the four codes of local slot ls (0 .. 1023) of a tile's code chunk held in shared memory.
 __device__ __forceinline__ void load_codes4_smem(const uint32_t *words, int ls, int bits, uint32_t c[4])
 {
@@ -143,7 +153,7 @@ __device__ __forceinline__ bool compute_all(bool ok)
 template <int MODE, int QW, int QS, bool FULL>
 __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
                                                    uint64_t *empty, int Lw, float Lwf, const float *utab,
-                                                   TileSmem &sm)
+                                                   float *ptab, TileSmem &sm)
 {
     const StagePlan &P = a.plan;
     const int64_t d = a.d;
@@ -151,23 +161,51 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
     const float nf = static_cast<float>(a.n);
     const bool pow2n = (a.n & (a.n - 1)) == 0;
     const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
-    float acc[kSlots][4];
-#pragma unroll
-    for (int k = 0; k < kSlots; ++k)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+    float acc[kSlots][4];  // the average of the decoded worker messages
     const float *sc = reinterpret_cast<const float *>(st + P.off_scales);
-#pragma unroll 4
-    for (int w = 0; w < a.n; ++w) {
-        const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
-        const float sw = has_scale<QW>() ? sc[w] : 0.0f;
+    if (QW == QK_SIGN && a.n <= 8) {
+        // Scaled-sign workers, n <= 8: a coordinate's average depends only on its n sign bits.
+        // Thread p forms the worker-order sum for sign pattern p, exactly as the per-coordinate
+        // loop would, divides by n, and the coordinates look their average up.
+        if (threadIdx.x < (1u << a.n)) {
+            float t = 0.0f;
+            for (int w = 0; w < a.n; ++w) t = __fadd_rn(t, ((threadIdx.x >> w) & 1u) ? sc[w] : -sc[w]);
+            ptab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
+        }
+        compute_sync();
+        const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
-            uint32_t c[4];
-            load_codes4_smem(cw, k * kThreads + threadIdx.x, bw, c);
+            const int wi = (k * kThreads + static_cast<int>(threadIdx.x)) >> 3;
+            uint32_t X = 0;  // bit 4w + i = worker w's code of coordinate i of the slot
+            for (int w = 0; w < a.n; ++w) {
+                const uint32_t word = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk)[wi];
+                X |= ((word >> sh) & 0xfu) << (4 * w);
+            }
 #pragma unroll
-            for (int i = 0; i < 4; ++i) acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
+            for (int i = 0; i < 4; ++i) acc[k][i] = ptab[gather_every4(X >> i)];
         }
+    } else {
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+#pragma unroll 4
+        for (int w = 0; w < a.n; ++w) {
+            const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
+            const float sw = has_scale<QW>() ? sc[w] : 0.0f;
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k) {
+                uint32_t c[4];
+                load_codes4_smem(cw, k * kThreads + threadIdx.x, bw, c);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[k][i] = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
     }
     // e_s (and m_s, v_s) are read from the stage only now, to keep registers for the sums
     float u[kSlots][4];
@@ -184,7 +222,7 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            float step = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
+            float step = acc[k][i];
             if (MODE == MODE_S) step = adam_step(step, ms[i], vs[i], a.hp);
             u[k][i] = (FULL || j0 + i < d) ? __fadd_rn(step, es[i]) : 0.0f;
         }
@@ -212,6 +250,7 @@ __global__ void __launch_bounds__(kThreads + 32, MODE == MODE_W ? 2 : 1) server_
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ TileSmem sm;
     __shared__ float utab[256];
+    __shared__ float ptab[256];  // scaled-sign workers: the average of every sign pattern
     const StagePlan &P = a.plan;
     const int S = P.stages;
     uint64_t *full = reinterpret_cast<uint64_t *>(dsm);
@@ -285,9 +324,9 @@ __global__ void __launch_bounds__(kThreads + 32, MODE == MODE_W ? 2 : 1) server_
         }
         const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
         if ((tile + 1) * kTile <= d)
-            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, sm);
+            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, ptab, sm);
         else
-            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, sm);
+            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, ptab, sm);
     }
 }
 

@@ -45,7 +45,7 @@ def test_ragged_sizes(d, group):
     _run_host(cfg, 3, seed=d)
 
 
-@pytest.mark.parametrize("n", [1, 2, 5])
+@pytest.mark.parametrize("n", [1, 2, 5, 8, 9, 16])
 def test_worker_counts(n):
     cfg = ea.EAConfig(d=9000, n=n, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-2)
     _run_host(cfg, 4, seed=n)
