@@ -138,6 +138,34 @@ int ea_get_view(const ea_handle *h, int32_t which, int32_t index, void **dev_ptr
 /* Synchronize the stream and report any asynchronous CUDA error or device-side check. */
 int ea_sync_status(ea_handle *h);
 
+/* Largest d accepted by ea_worker_compress_noalloc. */
+#define EA_NOALLOC_MAX_D ((int64_t)16384 * 4096)
+
+/* The paper has no counterpart: this is a deployment convenience.  Worker compress (the same
+ * computation as ea_worker_compress, with the same kernels) for callers that cannot allocate
+ * device memory -- code running inside a framework whose caching allocator has already reserved
+ * the GPU's memory, latency-critical paths that must not take cudaMalloc's implicit
+ * synchronisation, or plug-ins that are handed only the buffers they work on.  It needs no handle
+ * and no workspace: the caller passes the worker's state and message buffers, and the scratch of
+ * the two-pass scale (one partial norm per 4096-coordinate tile) is a fixed 128 KB array in device
+ * memory compiled into the library, which every GPU that loads the library holds until the process
+ * exits.  Nothing is allocated (no cudaMalloc/cudaFree, no library allocator).
+ *   - Only Q_w = EA_Q_SIGN_L1 or EA_Q_UNIFORM_MAX with one scale for the whole vector (group 0);
+ *     other quantizers return EA_E_UNSUPPORTED.  cfg->qs is ignored.
+ *   - 1 <= d <= EA_NOALLOC_MAX_D (67,108,864); larger d returns EA_E_INVAL.
+ *   - g (read), m and v (Adam at the worker; ignored, may be NULL, with Adam at the server) and e
+ *     (read and written): device, d binary32 values, 16-byte aligned.  Start them at m = 0,
+ *     v = eps, e = 0 as Algorithm 2 does.  codes: device, 16-byte aligned, room for
+ *     4 * ceil(d * bits / 128) words; scales: device, one binary32.  round: the 0-based round,
+ *     which with `worker` and cfg->seed keys the stochastic rounding.  stream: a cudaStream_t.
+ *   - The first call on each device looks up the scratch array's device address (with that
+ *     device current); make that first call before any stream capture.
+ *   - Every call shares the one array, which keeps the last call's contents; the calls rewrite all
+ *     of it that they read.  Calls that overlap on the GPU race: order them on one stream or with
+ *     events. */
+int ea_worker_compress_noalloc(const ea_config *cfg, int32_t worker, int64_t round, const float *g, float *m,
+                               float *v, float *e, uint32_t *codes, float *scales, void *stream);
+
 /* Text of the last error on h (or of the last handle-less failure when h is NULL). */
 const char *ea_last_error(const ea_handle *h);
 

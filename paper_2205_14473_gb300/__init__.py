@@ -30,7 +30,8 @@ EA_E_CUDA, EA_E_TIMEOUT, EA_E_DEVICE_CHECK, EA_E_UNSUPPORTED = -5, -6, -7, -8
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libea.so")
 EXPORTED = ["ea_workspace_bytes", "ea_init", "ea_worker_compress", "ea_server_step", "ea_worker_apply",
-            "ea_bits_sent", "ea_round_index", "ea_get_view", "ea_sync_status", "ea_last_error", "ea_destroy"]
+            "ea_bits_sent", "ea_round_index", "ea_get_view", "ea_sync_status", "ea_last_error", "ea_destroy",
+            "ea_worker_compress_noalloc"]
 
 
 class EAError(RuntimeError):
@@ -79,6 +80,7 @@ def lib() -> ctypes.CDLL:
             L.ea_last_error.argtypes = [_P]
             L.ea_last_error.restype = ctypes.c_char_p
             L.ea_destroy.argtypes = [_P]
+            L.ea_worker_compress_noalloc.argtypes = [C, ctypes.c_int32, ctypes.c_int64, _P, _P, _P, _P, _P, _P, _P]
             _lib = L
     return _lib
 
@@ -138,6 +140,13 @@ def ea_sync_status(h: int) -> None:
 
 def ea_destroy(h: int) -> None:
     lib().ea_destroy(h)
+
+
+def ea_worker_compress_noalloc(cfg: ea_config, worker: int, round_index: int, g_ptr: int, m_ptr: int, v_ptr: int,
+                               e_ptr: int, codes_ptr: int, scales_ptr: int, stream_ptr: int) -> None:
+    """Worker compress for callers that cannot allocate (see include/ea.h): no handle, no workspace."""
+    _check(lib().ea_worker_compress_noalloc(ctypes.byref(cfg), worker, round_index, g_ptr, m_ptr, v_ptr, e_ptr,
+                                            codes_ptr, scales_ptr, stream_ptr))
 
 
 # --------------------------------------------------------------------------- config marshalling

@@ -352,6 +352,8 @@ int second_pass(ea_handle *h, const QHost &q, float *buf, uint32_t *words, float
 
 }  // namespace
 
+void ea::set_last_error(const char *msg) { g_last_error = msg; }
+
 extern "C" {
 
 int ea_workspace_bytes(const ea_config *cfg, size_t *bytes)

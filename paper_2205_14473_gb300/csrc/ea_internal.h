@@ -130,4 +130,7 @@ cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s);
 cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s);
 cudaError_t launch_fill(float *p, int64_t count, float value, cudaStream_t s);
 
+// Record the text that ea_last_error(NULL) reports for a failure that has no handle.
+void set_last_error(const char *msg);
+
 }  // namespace ea
