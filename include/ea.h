@@ -95,8 +95,10 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
 /* Algorithm 2 for worker `worker` in the current round: with Adam at the worker,
  *   v <- theta v + (1-theta) g^2;  m <- beta m + (1-beta) g;  u = alpha m / sqrt(v) + e;
  * with Adam at the server, u = g + e.  Then send Q_w(u) (into the worker's message buffer) and
- * keep e <- u - Q_w(u).  g: device, d binary32 values, 16-byte aligned, read only, not retained.
- * Each worker compresses once per round; EA_E_ORDER otherwise. */
+ * keep e <- u - Q_w(u).  g: d binary32 values, 16-byte aligned, read only, not retained; device
+ * memory, or pinned host memory mapped into the device's address space (the kernel then reads it
+ * over the host link, with no staging copy).  Each worker compresses once per round; EA_E_ORDER
+ * otherwise. */
 int ea_worker_compress(ea_handle *h, int32_t worker, const float *g);
 
 /* Algorithm 1: average the n decoded worker messages (summed in worker order, then divided by
