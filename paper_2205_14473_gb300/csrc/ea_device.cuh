@@ -338,12 +338,20 @@ __device__ __forceinline__ uint32_t spread8_by4(uint32_t x)
 // called by all 32 lanes of the warp.  Codes of coordinates >= d are 0 (caller's job).
 // b = 1: one ballot per component; lanes 8g .. 8g+7 fill word (q_lane0 / 8) + g, whose bit
 // 4l + c is component c of lane 8g + l.
-template <bool FULL = false>
+template <bool FULL = false, bool BALLOT = true>
 __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64_t q, int bits, const uint32_t c[4],
                                              int64_t n_words)
 {
     const int lane = threadIdx.x & 31;
-    if (bits == 1) {
+    if (bits == 1 && !BALLOT) {
+        // b = 1 with three shuffles: lane l's nibble goes to bits 4(l mod 8) of its 8-lane word
+        uint32_t v = (c[0] | (c[1] << 1) | (c[2] << 2) | (c[3] << 3)) << (4 * (lane & 7));
+        v |= __shfl_xor_sync(0xffffffffu, v, 1);
+        v |= __shfl_xor_sync(0xffffffffu, v, 2);
+        v |= __shfl_xor_sync(0xffffffffu, v, 4);
+        const int64_t wi = q >> 3;
+        if ((lane & 7) == 0 && (FULL || wi < n_words)) words[wi] = v;
+    } else if (bits == 1) {
         const uint32_t b0 = __ballot_sync(0xffffffffu, c[0] != 0);
         const uint32_t b1 = __ballot_sync(0xffffffffu, c[1] != 0);
         const uint32_t b2 = __ballot_sync(0xffffffffu, c[2] != 0);

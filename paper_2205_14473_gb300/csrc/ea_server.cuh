@@ -166,24 +166,29 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
     if (QW == QK_SIGN && a.n <= 8) {
         // Scaled-sign workers, n <= 8: a coordinate's average depends only on its n sign bits.
         // Thread p forms the worker-order sum for sign pattern p, exactly as the per-coordinate
-        // loop would, divides by n, and the coordinates look their average up.
-        if (threadIdx.x < (1u << a.n)) {
+        // loop would, divides by n, and the coordinates look their average up.  The pattern of
+        // coordinate i of a slot is gathered from X (bit 4w + i = worker w's code) by one multiply:
+        // ((X >> i) & 0x11111111) * 0x01020408 carries no bits and leaves worker w's code at bit
+        // 24 + pi(w), pi = (0, 4, 1, 5, 2, 6, 3, 7); the table is indexed in that order.
+        if (threadIdx.x < 256) {
+            constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
             float t = 0.0f;
-            for (int w = 0; w < a.n; ++w) t = __fadd_rn(t, ((threadIdx.x >> w) & 1u) ? sc[w] : -sc[w]);
+            for (int w = 0; w < a.n; ++w)
+                t = __fadd_rn(t, ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? sc[w] : -sc[w]);
             ptab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
         }
         compute_sync();
         const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
+        const uint32_t *c0 = reinterpret_cast<const uint32_t *>(st + P.off_codes);
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
             const int wi = (k * kThreads + static_cast<int>(threadIdx.x)) >> 3;
             uint32_t X = 0;  // bit 4w + i = worker w's code of coordinate i of the slot
-            for (int w = 0; w < a.n; ++w) {
-                const uint32_t word = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk)[wi];
-                X |= ((word >> sh) & 0xfu) << (4 * w);
-            }
 #pragma unroll
-            for (int i = 0; i < 4; ++i) acc[k][i] = ptab[gather_every4(X >> i)];
+            for (int w = 0; w < 8; ++w)
+                if (w < a.n) X |= ((c0[w * (kTile / 32) + wi] >> sh) & 0xfu) << (4 * w);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[k][i] = ptab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
         }
     } else {
 #pragma unroll
@@ -234,8 +239,8 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
     // the stage is no longer read: hand it back to the producer before the tile's epilogue
     __syncwarp();
     if ((threadIdx.x & 31) == 0) mbar_arrive(empty);
-    finish_tile<QS, FULL>(u, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.pass, a.seed,
-                          static_cast<uint32_t>(a.n), a.t, a.partials, sm);
+    finish_tile<QS, FULL, false>(u, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.pass, a.seed,
+                                 static_cast<uint32_t>(a.n), a.t, a.partials, sm);
 }
 
 // The server's round with its inputs staged through shared memory.  Persistent CTAs of 8 compute

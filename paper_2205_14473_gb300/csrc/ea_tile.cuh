@@ -23,7 +23,7 @@ __device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
 
 // Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
 // FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
-template <int QK, bool FULL>
+template <int QK, bool FULL, bool BALLOT = true>
 __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
                                              const QParams &q, uint32_t *words, float *resid, int ef,
                                              uint64_t seed, uint32_t id, uint32_t t)
@@ -46,7 +46,7 @@ __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int
             c[i] = (FULL || j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec) : 0u;
             e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;
         }
-        store_codes4<FULL>(words, qs, bits, c, n_words);
+        store_codes4<FULL, BALLOT>(words, qs, bits, c, n_words);
         if (ef && (FULL || j0 < d)) store4<FULL>(resid, qs, d, e);
     }
 }
@@ -54,14 +54,16 @@ __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int
 // The tile's end for a quantizer with scale groups.
 //   PASS_FUSED: the tile is exactly one scale group (blocks of 4096): reduce, encode, store.
 //   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
-template <int QK, bool FULL = false>
+// BALLOT: pack 1-bit codes with __ballot_sync (worker kernels) or with shuffles (the server, whose
+// tile loop is instruction-bound).
+template <int QK, bool FULL = false, bool BALLOT = true>
 __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile, int64_t d, const QParams &q,
                                             uint32_t *words, float *scales, float *resid, int ef, int pass,
                                             uint64_t seed, uint32_t id, uint32_t t, double *partials,
                                             TileSmem &sm)
 {
     if constexpr (!has_scale<QK>()) {
-        encode_store<QK, FULL>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t);
+        encode_store<QK, FULL, BALLOT>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t);
         return;
     } else {
         const int64_t tile_lo = tile * kTile;
@@ -84,7 +86,7 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
                 s = block_max_all(mx, sm.redm);
             }
             if (threadIdx.x == 0) scales[tile] = s;
-            encode_store<QK, FULL>(u, s, tile, d, q, words, resid, ef, seed, id, t);
+            encode_store<QK, FULL, BALLOT>(u, s, tile, d, q, words, resid, ef, seed, id, t);
             return;
         }
         // PASS_STASH

@@ -115,33 +115,51 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
     }
 }
 
-// x <- x - Q_s(w): decode the broadcast and update x (Algorithm 1 and Algorithm 2).
+// x <- x - Q_s(w) on one 4096-coordinate tile (Algorithm 1 and Algorithm 2): all loads of the
+// tile are issued first; with 4096-block scales the tile has one scale.
 // HBM traffic per coordinate: 4 B read + 4 B written + b/8 B of code.
+template <int QK, bool FULL>
+__device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile)
+{
+    const int64_t d = a.d;
+    const Grouping &G = a.q.grp;
+    const int bits = code_bits<QK>(a.q);
+    const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
+    const float Lf = static_cast<float>(L);
+    float x[kSlots][4];
+    uint32_t c[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        load4<FULL>(a.x, q, d, x[k]);
+        if (FULL || 4 * q < d) load_codes4(a.words, q, bits, c[k]);
+    }
+    const bool tile_scale = G.gkind == GK_BLOCK && G.G == kTile;
+    const float s_tile = (has_scale<QK>() && tile_scale) ? __ldg(a.scales + tile) : 0.0f;
+    const int64_t hint = first_group_of_tile(G, tile);
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        const int64_t j0 = 4 * q;
+        if (!FULL && j0 >= d) continue;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (FULL || j0 + i < d) {
+                float s = s_tile;
+                if (has_scale<QK>() && !tile_scale) s = __ldg(a.scales + group_of(G, j0 + i, hint));
+                x[k][i] = __fsub_rn(x[k][i], decode1<QK>(c[k][i], s, a.q, Lf, L, nullptr));
+            }
+        }
+        store4<FULL>(a.x, q, d, x[k]);
+    }
+}
+
 template <int QK>
 __global__ void __launch_bounds__(kThreads) apply_kernel(const ApplyArgs a)
 {
-    const int64_t d = a.d;
-    const int64_t n_slots = (d + 3) >> 2;
-    const Grouping &G = a.q.grp;
-    const int L = (QK == QK_UNIF) ? unif_L(a.q.bits) : 0;
-    const float Lf = static_cast<float>(L);
-    for (int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; q < n_slots;
-         q += static_cast<int64_t>(gridDim.x) * kThreads) {
-        const int64_t j0 = 4 * q;
-        float x[4];
-        load4(a.x, q, d, x);
-        uint32_t c[4];
-        load_codes4(a.words, q, a.q.bits, c);
-        const int64_t hint = first_group_of_tile(G, j0 / kTile);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if (j0 + i < d) {
-                const float s = has_scale<QK>() ? a.scales[group_of(G, j0 + i, hint)] : 0.0f;
-                x[i] = __fsub_rn(x[i], decode1<QK>(c[i], s, a.q, Lf, L, nullptr));
-            }
-        }
-        store4(a.x, q, d, x);
-    }
+    const int64_t tile = blockIdx.x;
+    if ((tile + 1) * kTile <= a.d) apply_tile<QK, true>(a, tile);
+    else apply_tile<QK, false>(a, tile);
 }
 
 __global__ void fill_kernel(float *p, int64_t count, float value)
@@ -189,9 +207,7 @@ cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s)
 
 cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s)
 {
-    const int64_t n_slots = (a.d + 3) >> 2;
-    const int64_t want = (n_slots + kThreads - 1) / kThreads;
-    const dim3 grid(static_cast<unsigned>(want < 152 * 32 ? want : 152 * 32)), block(kThreads);
+    const dim3 grid(static_cast<unsigned>((a.d + kTile - 1) / kTile)), block(kThreads);
     switch (a.q.kind) {
     case QK_SIGN: apply_kernel<QK_SIGN><<<grid, block, 0, s>>>(a); break;
     case QK_UNIF: apply_kernel<QK_UNIF><<<grid, block, 0, s>>>(a); break;
