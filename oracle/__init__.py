@@ -52,7 +52,7 @@ class _Quant(ctypes.Structure):
 
 class _Config(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int64), ("n", ctypes.c_int32), ("mode", ctypes.c_int32),
-                ("error_feedback", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("error_feedback", ctypes.c_int32), ("adam_form", ctypes.c_int32),
                 ("alpha", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
                 ("eps", ctypes.c_float), ("seed", ctypes.c_uint64)]
 
@@ -82,6 +82,8 @@ def lib():
                                           ctypes.POINTER(_Quant), _P, ctypes.c_uint32, _P, _P, _P, _P,
                                           _P, _P, _P, _P, _P, _P]
             L.ora_apply.argtypes = [ctypes.POINTER(_Quant), ctypes.c_int64, _P, _P, _P, _P]
+            L.ora_bias_correction.argtypes = [ctypes.c_float, ctypes.c_uint32]
+            L.ora_bias_correction.restype = ctypes.c_float
             _lib = L
     return _lib
 
@@ -170,21 +172,22 @@ class OracleRound:
 
     def __init__(self, d: int, n: int, qw: Quantizer, qs: Quantizer, alpha: float, beta1: float,
                  beta2: float, eps: float, seed: int = 0, mode: int = ADAM_AT_WORKER,
-                 error_feedback: bool = True, gidx=None, threads: int = 1):
+                 error_feedback: bool = True, gidx=None, threads: int = 1, adam_form: int = 0):
         self.d, self.n, self.qw, self.qs, self.mode = d, n, qw, qs, mode
-        self.cfg = _Config(d, n, mode, int(error_feedback), 0, np.float32(alpha), np.float32(beta1),
+        self.cfg = _Config(d, n, mode, int(error_feedback), int(adam_form), np.float32(alpha), np.float32(beta1),
                            np.float32(beta2), np.float32(eps), seed)
+        v0 = np.float32(eps) if adam_form == 0 else np.float32(0.0)  # the textbook form starts v at 0
         f32 = np.float32
         self.e = np.zeros((n, d), f32)
         self.es = np.zeros(d, f32)
         if mode == ADAM_AT_WORKER:  # Algorithm 2: m_0 = 0, v_0 = eps on every worker
             self.m = np.zeros((n, d), f32)
-            self.v = np.full((n, d), f32(eps), f32)
+            self.v = np.full((n, d), v0, f32)
             self.ms = self.vs = np.zeros(1, f32)
         else:
             self.m = self.v = np.zeros((n, 1), f32)
             self.ms = np.zeros(d, f32)
-            self.vs = np.full(d, f32(eps), f32)
+            self.vs = np.full(d, v0, f32)
         self.wwords = np.zeros((n, max(qw.n_words(d), 1)), np.uint32)
         self.wscales = np.zeros((n, max(qw.n_groups, 1)), f32)
         self.swords = np.zeros(max(qs.n_words(d), 1), np.uint32)
@@ -196,6 +199,10 @@ class OracleRound:
         self.threads = max(1, int(threads))
         self._scratch = [(np.zeros(d, f32), np.zeros(d, f32)) for _ in range(n)]
         self._sscratch = (np.zeros(d, f32), np.zeros(d, f32), np.zeros(d, f32))
+
+    def set_hparams(self, alpha: float, beta1: float, beta2: float) -> None:
+        """alpha_t, beta and theta_t for the following rounds (schedules such as Assumption 2's)."""
+        self.cfg.alpha, self.cfg.beta1, self.cfg.beta2 = np.float32(alpha), np.float32(beta1), np.float32(beta2)
 
     def worker_compress(self, i: int, g: np.ndarray) -> None:
         g = np.ascontiguousarray(g, dtype=np.float32)

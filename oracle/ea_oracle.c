@@ -14,6 +14,9 @@
  *     e_s <- w - Q_s(w), x <- x - Q_s(w).
  *   - A second placement in which the Adam moments live on the server (workers send Q_w(g + e)),
  *     selected by `mode`; the paper itself uses the first.
+ *   - alpha_t and theta_t may change between rounds (Assumption 2 sets them from T; the experiments
+ *     decay alpha in steps): the caller updates the config before a round.  A textbook Adam form
+ *     (bias correction, eps in the denominator, v_0 = 0) is selected by `adam_form`.
  *   - Quantizers: Example 1 (l_inf-scaled uniform grid, deterministic nearest point), the same grid
  *     with stochastic rounding driven by Philox4x32-10, Example 2 (nearest power of two), the scaled
  *     sign compressor of Definition 3 (scale = mean |u| of the group) and the 32-bit identity
@@ -276,18 +279,33 @@ typedef struct {
     int32_t n;
     int32_t mode;            /* ORA_ADAM_AT_WORKER (the paper) or ORA_ADAM_AT_SERVER */
     int32_t error_feedback;  /* 1: the paper; 0: the "_err" ablation of Table 2 (residuals stay 0) */
-    int32_t reserved;
+    int32_t adam_form;       /* 0: the paper's Adam (Algorithm 2); 1: the textbook form below */
     float alpha, beta1, beta2, eps;
     uint64_t seed;
 } ora_config;
 
-/* One Adam moment update in the paper's form (Algorithm 2): no bias correction, eps only as v_0. */
-static float adam_step(float g, float *m, float *v, float alpha, float beta1, float beta2)
+/* 1 - beta^t for the 1-based round t, with beta^t formed by t binary64 multiplications and
+ * rounded once to binary32. */
+float ora_bias_correction(float beta, uint32_t t1)
 {
-    const float c1 = 1.0f - beta1, c2 = 1.0f - beta2;
-    *v = beta2 * *v + c2 * (g * g);
-    *m = beta1 * *m + c1 * g;
-    return (alpha * *m) / sqrtf(*v);
+    double p = 1.0;
+    for (uint32_t k = 0; k < t1; ++k) p *= (double)beta;
+    return (float)(1.0 - p);
+}
+
+/* One Adam moment update and step at the 1-based round t1.
+ * Form 0, the paper's (Algorithm 2): v = theta v + (1-theta) g^2, m = beta m + (1-beta) g, step
+ *   alpha m / sqrt(v); no bias correction, eps only as v_0.
+ * Form 1, the textbook form of Kingma and Ba: the same moments from v_0 = 0, step
+ *   alpha (m / (1 - beta^t)) / (sqrt(v / (1 - theta^t)) + eps). */
+static float adam_step(const ora_config *c, uint32_t t1, float g, float *m, float *v)
+{
+    const float c1 = 1.0f - c->beta1, c2 = 1.0f - c->beta2;
+    *v = c->beta2 * *v + c2 * (g * g);
+    *m = c->beta1 * *m + c1 * g;
+    if (c->adam_form == 0) return (c->alpha * *m) / sqrtf(*v);
+    const float bc1 = ora_bias_correction(c->beta1, t1), bc2 = ora_bias_correction(c->beta2, t1);
+    return (c->alpha * (*m / bc1)) / (sqrtf(*v / bc2) + c->eps);
 }
 
 /*
@@ -301,9 +319,7 @@ void ora_worker_step(const ora_config *cfg, const ora_quant *qw, const int64_t *
 {
     const int64_t d = cfg->d;
     for (int64_t l = 0; l < d; ++l) {
-        const float step = (cfg->mode == ORA_ADAM_AT_WORKER)
-                               ? adam_step(g[l], &m[l], &v[l], cfg->alpha, cfg->beta1, cfg->beta2)
-                               : g[l];
+        const float step = (cfg->mode == ORA_ADAM_AT_WORKER) ? adam_step(cfg, t + 1, g[l], &m[l], &v[l]) : g[l];
         u[l] = step + e[l];
     }
     ora_quantize(qw, d, u, gidx, cfg->seed, (uint32_t)worker, t, words, scales, dec);
@@ -330,9 +346,7 @@ void ora_server_step(const ora_config *cfg, const ora_quant *qw, const ora_quant
     }
     for (int64_t l = 0; l < d; ++l) {
         const float avg = acc[l] / (float)cfg->n;
-        const float step = (cfg->mode == ORA_ADAM_AT_SERVER)
-                               ? adam_step(avg, &ms[l], &vs[l], cfg->alpha, cfg->beta1, cfg->beta2)
-                               : avg;
+        const float step = (cfg->mode == ORA_ADAM_AT_SERVER) ? adam_step(cfg, t + 1, avg, &ms[l], &vs[l]) : avg;
         w[l] = step + es[l];
     }
     ora_quantize(qs, d, w, gidx, cfg->seed, (uint32_t)cfg->n, t, swords, sscales, dec);

@@ -191,3 +191,57 @@ def test_no_error_feedback_ablation_keeps_residuals_zero():
         orc.compress_all([rng.standard_normal(d).astype(np.float32) for _ in range(n)])
         orc.server_step()
         assert np.all(orc.e == 0) and np.all(orc.es == 0)
+
+
+def test_textbook_form_reduces_to_torch_adam():
+    """adam_form = 1 (bias correction, eps in the denominator, v_0 = 0) with the 32-bit identity
+    quantizer is plain Adam: x follows torch.optim.Adam, a library implementation, within binary32
+    rounding (the two evaluate the same expression in different operation orders)."""
+    torch = pytest.importorskip("torch")
+    d, T = 300, 60
+    a, b1, b2, eps = _f(3e-3), _f(0.9), _f(0.99), _f(1e-3)  # eps comparable to sqrt(v^): it matters
+    orc = _round(d, 1, O.Q_IDENTITY, O.Q_IDENTITY, 32, 32, alpha=a, beta1=b1, beta2=b2, eps=eps, adam_form=1)
+    rng = np.random.default_rng(21)
+    x0 = rng.standard_normal(d).astype(np.float32)
+    x = x0.copy()
+    p = torch.nn.Parameter(torch.from_numpy(x0.copy()))
+    opt = torch.optim.Adam([p], lr=a, betas=(b1, b2), eps=eps, foreach=False)
+    for t in range(T):
+        g = (rng.standard_normal(d) * 10 ** rng.uniform(-4, 0)).astype(np.float32)
+        orc.compress_all([g])
+        orc.server_step()
+        orc.apply(x)
+        p.grad = torch.from_numpy(g.copy())
+        opt.step()
+        np.testing.assert_allclose(x, p.detach().numpy(), rtol=2e-6, atol=a * 2e-5 * (t + 1))
+    assert np.abs(x - x0).max() > 10 * a  # it moved
+
+
+def test_schedules_follow_the_product_form():
+    """alpha_t, beta and theta_t changed every round (Assumption 2 fixes them from T; the experiments
+    decay alpha in steps).  With the identity quantizer the paper's moments are the product-form
+    sums  v_t = (prod_{j<=t} theta_j) eps + sum_{k<=t} (prod_{k<j<=t} theta_j) (1 - theta_k) g_k^2
+    and   m_t = sum_{k<=t} (prod_{k<j<=t} beta_j) (1 - beta_k) g_k,  and x moves by alpha_t m_t/sqrt(v_t)."""
+    d, T = 200, 40
+    eps = _f(1e-8)
+    orc = _round(d, 1, O.Q_IDENTITY, O.Q_IDENTITY, 32, 32, alpha=1e-2, beta1=0.9, beta2=0.99, eps=eps)
+    rng = np.random.default_rng(8)
+    x = np.zeros(d, np.float32)
+    xr = np.zeros(d)
+    al, be, th, G = [], [], [], []
+    for t in range(1, T + 1):
+        al.append(_f(1e-2 / np.sqrt(t)))
+        be.append(_f(0.9 - 0.3 * (t % 3 == 0)))
+        th.append(_f(1 - 0.5 / (t + 1)))
+        orc.set_hparams(al[-1], be[-1], th[-1])
+        g = rng.standard_normal(d).astype(np.float32)
+        G.append(g.astype(np.float64))
+        orc.compress_all([g])
+        orc.server_step()
+        orc.apply(x)
+        v = np.prod(th) * eps + sum(np.prod(th[k + 1:]) * (1 - th[k]) * G[k] ** 2 for k in range(t))
+        m = sum(np.prod(be[k + 1:]) * (1 - be[k]) * G[k] for k in range(t))
+        xr = xr - al[-1] * m / np.sqrt(v)
+        np.testing.assert_allclose(orc.v[0], v, rtol=4e-7 * t + 1e-6)
+        assert np.all(np.abs(orc.m[0] - m) <= (4e-7 * t + 1e-6) * np.max(np.abs(G[: t]), axis=0))
+        np.testing.assert_allclose(x, xr, rtol=1e-5, atol=1e-7 * t)
