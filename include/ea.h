@@ -70,12 +70,14 @@ typedef struct ea_config {
     int32_t placement;    /* ea_placement */
     ea_quantizer qw;      /* Q_w, the workers' mapping (Algorithm 2) */
     ea_quantizer qs;      /* Q_s, the server's mapping (Algorithm 1) */
-    float alpha;          /* alpha_t (constant; see ea_set_hparams for schedules) */
+    float alpha;          /* alpha_t (ea_set_hparams changes it between rounds) */
     float beta1;          /* beta, the first-moment coefficient, 0 <= beta1 < 1 */
     float beta2;          /* theta_t, the second-moment coefficient, 0 <= beta2 < 1 */
-    float eps;            /* v_0 = eps (Algorithm 2); no eps in the denominator, no bias correction */
+    float eps;            /* adam_form 0: v_0 = eps (Algorithm 2), no eps in the denominator, no bias
+                             correction; adam_form 1: v_0 = 0 and eps added to the denominator */
     int32_t error_feedback; /* 1 = the paper; 0 = the "_err" ablation of Table 2 */
-    int32_t reserved;     /* must be 0 */
+    int32_t adam_form;    /* 0 = the paper's Adam (Algorithm 2); 1 = the textbook form, step
+                             alpha (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + eps), t 1-based */
     uint64_t seed;        /* Philox key for stochastic rounding */
 } ea_config;
 
@@ -111,6 +113,11 @@ int ea_server_step(ea_handle *h);
  * x: device, d binary32 values, 16-byte aligned, updated in place.  Call once per replica of x.
  * EA_E_ORDER before the first ea_server_step. */
 int ea_worker_apply(ea_handle *h, float *x);
+
+/* alpha_t, beta and theta_t (= beta2) for the calls that follow, e.g. between rounds: Assumption 2
+ * sets theta_t = 1 - theta/T and alpha_t = alpha/sqrt(T) from the horizon T; the experiments decay
+ * alpha in steps.  Same ranges as ea_config; EA_E_INVAL otherwise (nothing changed). */
+int ea_set_hparams(ea_handle *h, float alpha, float beta1, float beta2);
 
 /* Cumulative bits sent (Corollary 1's accounting): up = per round n messages of d*b_w bits plus
  * 32 per scale word of Q_w; down = the broadcast counted once per receiving worker, n messages of
@@ -157,7 +164,7 @@ int ea_sync_status(ea_handle *h);
  *   - 1 <= d <= EA_NOALLOC_MAX_D (67,108,864); larger d returns EA_E_INVAL.
  *   - g (read), m and v (Adam at the worker; ignored, may be NULL, with Adam at the server) and e
  *     (read and written): device, d binary32 values, 16-byte aligned.  Start them at m = 0,
- *     v = eps, e = 0 as Algorithm 2 does.  codes: device, 16-byte aligned, room for
+ *     v = eps (0 with adam_form 1), e = 0 as Algorithm 2 does.  codes: device, 16-byte aligned, room for
  *     4 * ceil(d * bits / 128) words; scales: device, one binary32.  round: the 0-based round,
  *     which with `worker` and cfg->seed keys the stochastic rounding.  stream: a cudaStream_t.
  *   - The first call on each device looks up the scratch array's device address (with that

@@ -31,7 +31,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libea.so")
 EXPORTED = ["ea_workspace_bytes", "ea_init", "ea_worker_compress", "ea_server_step", "ea_worker_apply",
             "ea_bits_sent", "ea_round_index", "ea_get_view", "ea_sync_status", "ea_last_error", "ea_destroy",
-            "ea_worker_compress_noalloc"]
+            "ea_worker_compress_noalloc", "ea_set_hparams"]
 
 
 class EAError(RuntimeError):
@@ -50,7 +50,7 @@ class ea_config(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int64), ("n", ctypes.c_int32), ("placement", ctypes.c_int32),
                 ("qw", ea_quantizer), ("qs", ea_quantizer), ("alpha", ctypes.c_float),
                 ("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
-                ("error_feedback", ctypes.c_int32), ("reserved", ctypes.c_int32), ("seed", ctypes.c_uint64)]
+                ("error_feedback", ctypes.c_int32), ("adam_form", ctypes.c_int32), ("seed", ctypes.c_uint64)]
 
 
 _lock = threading.Lock()
@@ -80,6 +80,7 @@ def lib() -> ctypes.CDLL:
             L.ea_last_error.argtypes = [_P]
             L.ea_last_error.restype = ctypes.c_char_p
             L.ea_destroy.argtypes = [_P]
+            L.ea_set_hparams.argtypes = [_P, ctypes.c_float, ctypes.c_float, ctypes.c_float]
             L.ea_worker_compress_noalloc.argtypes = [C, ctypes.c_int32, ctypes.c_int64, _P, _P, _P, _P, _P, _P, _P]
             _lib = L
     return _lib
@@ -114,6 +115,10 @@ def ea_server_step(h: int) -> None:
 
 def ea_worker_apply(h: int, x_ptr: int) -> None:
     _check(lib().ea_worker_apply(h, x_ptr), h)
+
+
+def ea_set_hparams(h: int, alpha: float, beta1: float, beta2: float) -> None:
+    _check(lib().ea_set_hparams(h, alpha, beta1, beta2), h)
 
 
 def ea_bits_sent(h: int) -> tuple[int, int]:
@@ -164,6 +169,7 @@ class EAConfig:
     placement: int = ADAM_AT_WORKER
     error_feedback: bool = True
     seed: int = 0
+    adam_form: int = 0          # 0: the paper's Adam; 1: the textbook (bias-corrected) form
 
     @classmethod
     def from_workload(cls, w: Workload, **kw) -> "EAConfig":
@@ -185,7 +191,7 @@ class EAConfig:
                                 len(spec.segments) if spec.group < 0 else 0, spec.group, seg)
 
         c = ea_config(self.d, self.n, self.placement, q(self.qw), q(self.qs), self.alpha, self.beta1, self.beta2,
-                      self.eps, int(self.error_feedback), 0, self.seed)
+                      self.eps, int(self.error_feedback), int(self.adam_form), self.seed)
         return c, keep
 
 
@@ -234,6 +240,9 @@ class EARound:
         self.apply(x)
 
     # inspection
+    def set_hparams(self, alpha: float, beta1: float, beta2: float) -> None:
+        ea_set_hparams(self.h, alpha, beta1, beta2)
+
     def bits_sent(self) -> tuple[int, int]:
         return ea_bits_sent(self.h)
 

@@ -198,7 +198,7 @@ int validate(const ea_config *cfg, QHost &qw, QHost &qs)
         return fail(nullptr, EA_E_INVAL, "unknown placement %d", cfg->placement);
     if (cfg->error_feedback != 0 && cfg->error_feedback != 1)
         return fail(nullptr, EA_E_INVAL, "error_feedback is 0 or 1");
-    if (cfg->reserved != 0) return fail(nullptr, EA_E_INVAL, "reserved must be 0");
+    if (cfg->adam_form != 0 && cfg->adam_form != 1) return fail(nullptr, EA_E_INVAL, "adam_form is 0 or 1");
     if (!std::isfinite(cfg->alpha)) return fail(nullptr, EA_E_INVAL, "alpha must be finite");
     if (!(cfg->beta1 >= 0.0f && cfg->beta1 < 1.0f)) return fail(nullptr, EA_E_INVAL, "beta1 must be in [0, 1)");
     if (!(cfg->beta2 >= 0.0f && cfg->beta2 < 1.0f)) return fail(nullptr, EA_E_INVAL, "beta2 must be in [0, 1)");
@@ -319,6 +319,25 @@ StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs,
     return P;
 }
 
+// The hyper-parameters of the current round (1-based t = h->t + 1 for the bias corrections).
+Hyper round_hyper(const ea_handle *h)
+{
+    Hyper hp = h->hp;
+    if (hp.form == 1) {
+        hp.bc1 = bias_correction(hp.beta1, h->t + 1);
+        hp.bc2 = bias_correction(hp.beta2, h->t + 1);
+    }
+    return hp;
+}
+
+int check_hparams(float alpha, float beta1, float beta2)
+{
+    if (!std::isfinite(alpha)) return fail(nullptr, EA_E_INVAL, "alpha must be finite");
+    if (!(beta1 >= 0.0f && beta1 < 1.0f)) return fail(nullptr, EA_E_INVAL, "beta1 must be in [0, 1)");
+    if (!(beta2 >= 0.0f && beta2 < 1.0f)) return fail(nullptr, EA_E_INVAL, "beta2 must be in [0, 1)");
+    return EA_OK;
+}
+
 int check_dev_ptr(ea_handle *h, const void *p, const char *what)
 {
     if (!p) return fail(h, EA_E_INVAL, "%s is NULL", what);
@@ -397,6 +416,8 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->hp.beta2 = cfg->beta2;
     h->hp.c1 = 1.0f - cfg->beta1;
     h->hp.c2 = 1.0f - cfg->beta2;
+    h->hp.form = cfg->adam_form;
+    h->hp.eps = cfg->eps;
 
     char *p = static_cast<char *>(workspace);
     auto take = [&p](size_t n) {
@@ -427,13 +448,15 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
         h->splan = make_server_plan(*cfg, h->qw, h->qs, h->n_tiles, sms);
 
-    // Algorithm 2: m_0 = 0, v_0 = eps, e_1 = 0; Algorithm 1: e_1 = 0.  Messages start zeroed.
+    // Algorithm 2: m_0 = 0, v_0 = eps (0 in the textbook form), e_1 = 0; Algorithm 1: e_1 = 0.
+    // Messages start zeroed.
     cudaStream_t s = h->stream;
+    const float v0 = cfg->adam_form == 0 ? cfg->eps : 0.0f;
     r = check_cuda(h, cudaMemsetAsync(workspace, 0, need, s), "workspace clear");
     if (r == EA_OK && cfg->placement == EA_ADAM_AT_WORKER)
-        r = check_cuda(h, launch_fill(h->v, static_cast<int64_t>(cfg->n) * L.dpad, cfg->eps, s), "v_0 fill");
+        r = check_cuda(h, launch_fill(h->v, static_cast<int64_t>(cfg->n) * L.dpad, v0, s), "v_0 fill");
     if (r == EA_OK && cfg->placement == EA_ADAM_AT_SERVER)
-        r = check_cuda(h, launch_fill(h->vs, L.dpad, cfg->eps, s), "v_0 fill");
+        r = check_cuda(h, launch_fill(h->vs, L.dpad, v0, s), "v_0 fill");
     auto upload = [&](void *dst, const void *src, size_t n) {
         if (r == EA_OK && n) r = check_cuda(h, cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s), "table upload");
     };
@@ -472,7 +495,7 @@ int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
     a.q = device_quant(h->qw);
     a.words = h->wcodes + worker * h->lay.wcode_stride;
     a.scales = h->wscales + worker * h->lay.wscale_stride;
-    a.hp = h->hp;
+    a.hp = round_hyper(h);
     a.ef = h->cfg.error_feedback;
     a.pass = h->qw.pass;
     a.seed = h->cfg.seed;
@@ -508,7 +531,7 @@ int ea_server_step(ea_handle *h)
     a.es = h->es;
     a.ms = h->ms;
     a.vs = h->vs;
-    a.hp = h->hp;
+    a.hp = round_hyper(h);
     a.ef = h->cfg.error_feedback;
     a.pass = h->qs.pass;
     a.seed = h->cfg.seed;
@@ -545,6 +568,22 @@ int ea_worker_apply(ea_handle *h, float *x)
     a.words = h->scodes;
     a.scales = h->sscales;
     return check_cuda(h, launch_apply(a, h->stream), "apply launch");
+}
+
+int ea_set_hparams(ea_handle *h, float alpha, float beta1, float beta2)
+{
+    if (!h) return fail(nullptr, EA_E_INVAL, "handle is NULL");
+    const int r = check_hparams(alpha, beta1, beta2);
+    if (r != EA_OK) {
+        h->err = ea_last_error(nullptr);
+        return r;
+    }
+    h->hp.alpha = alpha;
+    h->hp.beta1 = beta1;
+    h->hp.beta2 = beta2;
+    h->hp.c1 = 1.0f - beta1;
+    h->hp.c2 = 1.0f - beta2;
+    return EA_OK;
 }
 
 int ea_bits_sent(const ea_handle *h, uint64_t *up_bits, uint64_t *down_bits)

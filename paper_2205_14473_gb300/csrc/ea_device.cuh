@@ -382,12 +382,16 @@ __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64
     }
 }
 
-// The paper's Adam moment update and step (Algorithm 2): no bias correction, eps only as v_0.
+// The Adam moment update and step.  Form 0, the paper's (Algorithm 2): no bias correction, eps
+// only as v_0, step alpha m / sqrt(v).  Form 1, the textbook one: v_0 = 0 and step
+// alpha (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + eps).
 __device__ __forceinline__ float adam_step(float g, float &m, float &v, const Hyper &h)
 {
     v = __fadd_rn(__fmul_rn(h.beta2, v), __fmul_rn(h.c2, __fmul_rn(g, g)));
     m = __fadd_rn(__fmul_rn(h.beta1, m), __fmul_rn(h.c1, g));
-    return __fdiv_rn(__fmul_rn(h.alpha, m), __fsqrt_rn(v));
+    if (h.form == 0) return __fdiv_rn(__fmul_rn(h.alpha, m), __fsqrt_rn(v));
+    const float mh = __fdiv_rn(m, h.bc1), vh = __fdiv_rn(v, h.bc2);
+    return __fdiv_rn(__fmul_rn(h.alpha, mh), __fadd_rn(__fsqrt_rn(vh), h.eps));
 }
 
 // ------------------------------------------------------------------------ vector helpers

@@ -36,7 +36,17 @@ struct QParams {
 
 struct Hyper {
     float alpha, beta1, beta2, c1, c2;  // c1 = 1 - beta1, c2 = 1 - beta2, rounded to binary32
+    int form;                           // 0: the paper's Adam (Algorithm 2); 1: the textbook form
+    float eps, bc1, bc2;                // textbook form: eps in the denominator, 1 - beta1^t, 1 - beta2^t
 };
+
+// 1 - beta^t for the 1-based round t: beta^t by t binary64 multiplications, rounded once.
+inline float bias_correction(float beta, int64_t t1)
+{
+    double p = 1.0;
+    for (int64_t k = 0; k < t1; ++k) p *= static_cast<double>(beta);
+    return static_cast<float>(1.0 - p);
+}
 
 // How the scale of a message is formed.
 enum Pass : int {

@@ -89,6 +89,7 @@ extern "C" int ea_worker_compress_noalloc(const ea_config *cfg, int32_t worker, 
     if (cfg->placement != EA_ADAM_AT_WORKER && cfg->placement != EA_ADAM_AT_SERVER)
         return fail(EA_E_INVAL, "unknown placement %d", cfg->placement);
     if (cfg->error_feedback != 0 && cfg->error_feedback != 1) return fail(EA_E_INVAL, "error_feedback is 0 or 1");
+    if (cfg->adam_form != 0 && cfg->adam_form != 1) return fail(EA_E_INVAL, "adam_form is 0 or 1");
     if (!std::isfinite(cfg->alpha) || !(cfg->beta1 >= 0.0f && cfg->beta1 < 1.0f) ||
         !(cfg->beta2 >= 0.0f && cfg->beta2 < 1.0f) || !(cfg->eps > 0.0f))
         return fail(EA_E_INVAL, "hyper-parameters out of range");
@@ -134,6 +135,12 @@ extern "C" int ea_worker_compress_noalloc(const ea_config *cfg, int32_t worker, 
     a.hp.beta2 = cfg->beta2;
     a.hp.c1 = 1.0f - cfg->beta1;
     a.hp.c2 = 1.0f - cfg->beta2;
+    a.hp.form = cfg->adam_form;
+    a.hp.eps = cfg->eps;
+    if (cfg->adam_form == 1) {
+        a.hp.bc1 = bias_correction(cfg->beta1, round + 1);
+        a.hp.bc2 = bias_correction(cfg->beta2, round + 1);
+    }
     a.ef = cfg->error_feedback;
     a.pass = d <= kTile ? PASS_FUSED : PASS_STASH;
     a.seed = cfg->seed;

@@ -89,10 +89,14 @@ class Lockstep:
         self.idx_dev = torch.from_numpy(self.idx).to(self.dev)
         self.orc = O.OracleRound(self.d_o, cfg.n, qw_o, qs_o, cfg.alpha, cfg.beta1, cfg.beta2, cfg.eps,
                                  seed=cfg.seed, mode=cfg.placement, error_feedback=cfg.error_feedback,
-                                 gidx=gidx, threads=threads)
+                                 gidx=gidx, threads=threads, adam_form=cfg.adam_form)
         self.tainted = torch.zeros(self.d_o, dtype=torch.bool, device=self.dev)
         self.total_mismatch = 0
         self.reports: list[RoundReport] = []
+
+    def set_hparams(self, alpha: float, beta1: float, beta2: float) -> None:
+        self.gpu.set_hparams(alpha, beta1, beta2)
+        self.orc.set_hparams(alpha, beta1, beta2)
 
     # ------------------------------------------------------------------------------------ inputs
     def host(self, t_dev: torch.Tensor) -> np.ndarray:

@@ -217,3 +217,26 @@ def test_c5_sampled_blocks_all_rounds(placement):
     assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (125_613_752_320, 125_613_752_320)
     del L, bufs, x_dev
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
+@pytest.mark.parametrize("form", [0, 1])
+@pytest.mark.parametrize("group", [4096, 0])
+def test_schedules_and_adam_forms(placement, form, group):
+    """alpha_t, beta and theta_t changed every round through ea_set_hparams (Assumption 2's
+    alpha/sqrt(T), 1 - theta/T and a step decay), in the paper's and the textbook Adam form."""
+    d = 13_000
+    cfg = ea.EAConfig(d=d, n=3, qw=W.sign_q(group), qs=W.uniform_q(8, group if group else 0, False), alpha=1e-2,
+                      placement=placement, adam_form=form, eps=1e-6, seed=3)
+    L = Lockstep(cfg)
+    rng = np.random.default_rng(17)
+    x_host = rng.standard_normal(d).astype(np.float32)
+    x_dev = torch.from_numpy(x_host.copy()).cuda()
+    T = 6
+    for t in range(1, T + 1):
+        L.set_hparams(1e-2 / np.sqrt(t) * (0.2 if t > 4 else 1.0), 0.9 - 0.2 * (t % 2), 1 - 0.1 / t)
+        gs = [(rng.standard_normal(d) * 10 ** rng.uniform(-3, 0)).astype(np.float32) for _ in range(cfg.n)]
+        L.round([torch.from_numpy(g).cuda() for g in gs], gs, x_dev, x_host)
+    with pytest.raises(ea.EAError) as ex:
+        L.gpu.set_hparams(1e-2, 1.0, 0.9)
+    assert ex.value.status == ea.EA_E_INVAL
