@@ -201,3 +201,43 @@ def sample_blocks(w: Workload, count: int, block: int = 4096) -> np.ndarray:
     rest = _rng(w.seed, "sample").choice(np.arange(1, max(nb - 1, 1)), size=max(0, min(count - 2, nb - 2)),
                                          replace=False)
     return np.unique(np.concatenate([[0, nb - 1], rest]).astype(np.int64))
+
+
+# ------------------------------------------------------------------- Section 5.1's convex toy
+# min_x E || A x - (x* + xi) ||^2 with A in R^{500 x 500}, A_ij ~ N(0, 1), x* ~ N(0, 0.1 I),
+# xi ~ N(0, 0.1 I), 10 workers, beta = 0.9, theta = 0.99; quantizers Example 1 with k = 1 ("com1")
+# and Example 2 with k = -17, K = -11 ("com2"); "full" is the 32-bit identity.
+
+TOY_D, TOY_N = 500, 10
+TOY_QUANTIZERS = {
+    "full": QuantSpec(Q_IDENTITY, 32, 0),
+    "com1": QuantSpec(Q_UNIFORM_MAX, 2, 0),
+    "com2": QuantSpec(Q_POW2, 4, 0, (), False, -17, -11),
+}
+
+
+def toy_case(case: int, d: int = TOY_D):
+    """A random case of the toy: (A, x*) in float32 and a generator for the noise draws."""
+    r = _rng(2051, "toy", case)
+    A = r.standard_normal((d, d), dtype=np.float32)
+    xs = (r.standard_normal(d, dtype=np.float32) * np.float32(np.sqrt(0.1))).astype(np.float32)
+    return A, xs
+
+
+def toy_noise(case: int, i: int, t: int, d: int = TOY_D) -> np.ndarray:
+    return (_rng(2051, "toy-xi", case, i, t).standard_normal(d, dtype=np.float32) *
+            np.float32(np.sqrt(0.1))).astype(np.float32)
+
+
+def toy_gradient(A: np.ndarray, x: np.ndarray, xs: np.ndarray, xi: np.ndarray) -> np.ndarray:
+    """The stochastic gradient 2 A^T (A x - x* - xi) of the toy (formed in binary64, rounded to
+    binary32), for any x (numpy)."""
+    A64 = A.astype(np.float64)
+    r = A64 @ x.astype(np.float64) - xs.astype(np.float64) - xi.astype(np.float64)
+    return (2.0 * (A64.T @ r)).astype(np.float32)
+
+
+def toy_full_gradient_norm(A: np.ndarray, x: np.ndarray, xs: np.ndarray) -> float:
+    """|| grad F(x) || = || 2 A^T (A x - x*) ||, the quantity Figure 2 plots."""
+    A64 = A.astype(np.float64)
+    return float(np.linalg.norm(2.0 * (A64.T @ (A64 @ x.astype(np.float64) - xs.astype(np.float64)))))

@@ -240,3 +240,24 @@ def test_schedules_and_adam_forms(placement, form, group):
     with pytest.raises(ea.EAError) as ex:
         L.gpu.set_hparams(1e-2, 1.0, 0.9)
     assert ex.value.status == ea.EA_E_INVAL
+
+
+@pytest.mark.parametrize("name", ["full", "com1", "com2"])
+@pytest.mark.parametrize("ef", [True, False])
+def test_toy_section51_lockstep(name, ef):
+    """Section 5.1's toy (500 x 500 Gaussian A, 10 workers, beta 0.9, theta 0.99) with its three
+    quantizer settings; each side forms 2 A^T (A x - x* - xi) from its own x."""
+    A, xs = W.toy_case(0)
+    spec = W.TOY_QUANTIZERS[name]
+    cfg = ea.EAConfig(d=W.TOY_D, n=W.TOY_N, qw=spec, qs=spec, alpha=1e-4, beta1=0.9, beta2=0.99,
+                      error_feedback=ef)
+    L = Lockstep(cfg)
+    x_dev = torch.zeros(W.TOY_D, device="cuda")
+    x_host = np.zeros(W.TOY_D, np.float32)
+    for t in range(40):
+        xi = [W.toy_noise(0, i, t) for i in range(W.TOY_N)]
+        xg = x_dev.cpu().numpy()
+        g_dev = [torch.from_numpy(W.toy_gradient(A, xg, xs, xi[i])).cuda() for i in range(W.TOY_N)]
+        g_host = [W.toy_gradient(A, x_host, xs, xi[i]) for i in range(W.TOY_N)]
+        L.round(g_dev, g_host, x_dev, x_host)
+    assert W.toy_full_gradient_norm(A, x_host, xs) < W.toy_full_gradient_norm(A, np.zeros_like(x_host), xs)
