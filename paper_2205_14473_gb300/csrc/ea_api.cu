@@ -281,9 +281,7 @@ uint64_t message_bits(const QHost &q, int64_t d)
 
 // Shared-memory staging of the server's inputs (see server_staged_kernel): one stage holds a
 // tile's e_s (+ m_s, v_s) and the n workers' code chunks and scales.  Enabled when both messages
-// have one scale per 4096-tile (or none) and a stage fits the budget: 100 KB per CTA and two CTAs
-// per SM with Adam at the workers; 200 KB and one CTA per SM (more registers) with Adam at the
-// server, whose stages are larger.
+// have one scale per 4096-tile (or none) and two stages fit in 200 KB.
 StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs, int64_t n_tiles, int sms)
 {
     StagePlan P{};
@@ -300,20 +298,23 @@ StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs,
         P.off_c = off;
         off += 4 * kTile;
     }
-    const uint32_t budget = server_adam ? 200 * 1024 : 100 * 1024;
+    // Two CTAs per SM when two stages fit 100 KB (106 KB with Adam at the server, whose stages hold
+    // m_s and v_s too); otherwise one CTA per SM with up to 200 KB of stages.
     P.code_chunk = static_cast<uint32_t>(kTile / 8 * qw.bits);
     P.off_codes = off;
     const uint64_t codes = static_cast<uint64_t>(P.code_chunk) * c.n;
-    if (codes > budget / 2) return P;
+    if (codes > 100 * 1024) return P;
     off += static_cast<uint32_t>(codes);
     P.off_scales = off;
     off += static_cast<uint32_t>(align_up(4 * static_cast<size_t>(c.n), 16));
     P.stage_bytes = static_cast<uint32_t>(align_up(off, 128));
+    const uint32_t two_cta = server_adam ? 106 * 1024 : 100 * 1024;
+    const uint32_t budget = (2 * P.stage_bytes <= two_cta) ? two_cta : 200 * 1024;
     if (2 * P.stage_bytes > budget) return P;
     P.stages = std::max(2, std::min(6, static_cast<int>(budget / P.stage_bytes)));
     const uint32_t bars = static_cast<uint32_t>(align_up(2 * 8 * static_cast<size_t>(P.stages), 128));
     P.smem_bytes = bars + static_cast<uint32_t>(P.stages) * P.stage_bytes;
-    const int per_sm = (!server_adam && 2 * (P.smem_bytes + 4096) <= 228 * 1024) ? 2 : 1;
+    const int per_sm = (2 * (P.smem_bytes + 8 * 1024) <= 228 * 1024) ? 2 : 1;  // + static shared memory
     P.grid = static_cast<int>(std::min<int64_t>(n_tiles, static_cast<int64_t>(sms) * per_sm));
     P.enabled = 1;
     return P;

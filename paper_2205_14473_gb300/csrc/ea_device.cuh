@@ -213,8 +213,10 @@ __device__ __forceinline__ float pow2_value(uint32_t code, int k, int bits)
 }
 
 // Encode one coordinate, returning the code and the decoded value Q(u).
+// qtab (may be null): fl(i / L) for i = -L .. L at qtab[i + L], the same values the division gives.
 template <int QK>
-__device__ __forceinline__ uint32_t encode1(float u, float s, const QParams &q, float Lf, int L, float U, float &dec)
+__device__ __forceinline__ uint32_t encode1(float u, float s, const QParams &q, float Lf, int L, float U, float &dec,
+                                            const float *qtab = nullptr)
 {
     if constexpr (QK == QK_SIGN) {
         const bool pos = u >= 0.0f;
@@ -222,7 +224,7 @@ __device__ __forceinline__ uint32_t encode1(float u, float s, const QParams &q, 
         return pos ? 1u : 0u;
     } else if constexpr (QK == QK_UNIF) {
         const int qi = unif_index(u, s, Lf, q.stochastic != 0, U);
-        dec = __fmul_rn(s, __fdiv_rn(static_cast<float>(qi), Lf));
+        dec = __fmul_rn(s, qtab ? qtab[qi + L] : __fdiv_rn(static_cast<float>(qi), Lf));
         return static_cast<uint32_t>(qi + L);
     } else if constexpr (QK == QK_POW2) {
         const uint32_t c = pow2_code(u, q.pow2_k, q.pow2_K, q.bits);
@@ -254,6 +256,18 @@ template <int QK>
 __device__ __forceinline__ constexpr bool has_scale()
 {
     return QK == QK_SIGN || QK == QK_UNIF;
+}
+
+// The uniform grid's fl(i / L), i = -L .. L, into tab[0 .. 2L] (no barrier; the caller orders it).
+// Returns tab, or null when the grid has more than 8 bits (then the division is used directly).
+template <int QK>
+__device__ __forceinline__ const float *build_qtab(const QParams &q, float *tab)
+{
+    if (QK != QK_UNIF || q.bits > 8) return nullptr;
+    const int L = (1 << (q.bits - 1)) - 1;
+    for (int i = threadIdx.x; i <= 2 * L; i += blockDim.x)
+        tab[i] = __fdiv_rn(static_cast<float>(i - L), static_cast<float>(L));
+    return tab;
 }
 
 // Code width: fixed by the kind for the sign (1) and identity (32) mappings, else configured.

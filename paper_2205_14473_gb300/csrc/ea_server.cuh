@@ -22,6 +22,7 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
     const int Lw = (QW == QK_UNIF) ? unif_L(a.qw.bits) : 0;
     const float Lwf = static_cast<float>(Lw);
     const bool use_tab = QW == QK_UNIF && a.qw.bits <= 8;
+    build_qtab<QS>(a.qs, sm.qtab);  // read after the scale reduction's barrier
     if (use_tab) {
         for (int i = threadIdx.x; i <= 2 * Lw; i += kThreads)
             utab[i] = __fdiv_rn(static_cast<float>(i - Lw), Lwf);
@@ -98,6 +99,8 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
 }
 
 
+constexpr int kWorkerTab = 1024;  // floats of the staged server's per-tile worker table
+
 // Bits 0, 4, ..., 28 of x moved to bits 0 .. 7 (the inverse of spread8_by4).
 __device__ __forceinline__ uint32_t gather_every4(uint32_t x)
 {
@@ -153,7 +156,7 @@ __device__ __forceinline__ bool compute_all(bool ok)
 template <int MODE, int QW, int QS, bool FULL>
 __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
                                                    uint64_t *empty, int Lw, float Lwf, const float *utab,
-                                                   float *ptab, TileSmem &sm)
+                                                   float *wtab, TileSmem &sm)
 {
     const StagePlan &P = a.plan;
     const int64_t d = a.d;
@@ -175,7 +178,7 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
             float t = 0.0f;
             for (int w = 0; w < a.n; ++w)
                 t = __fadd_rn(t, ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? sc[w] : -sc[w]);
-            ptab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
+            wtab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
         }
         compute_sync();
         const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
@@ -188,23 +191,36 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
             for (int w = 0; w < 8; ++w)
                 if (w < a.n) X |= ((c0[w * (kTile / 32) + wi] >> sh) & 0xfu) << (4 * w);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) acc[k][i] = ptab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
+            for (int i = 0; i < 4; ++i) acc[k][i] = wtab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
         }
     } else {
 #pragma unroll
         for (int k = 0; k < kSlots; ++k)
 #pragma unroll
             for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+        // Uniform-grid workers: every worker's 2L+1 decoded values s_w * fl(i/L) for this tile, as
+        // decode1 would form them, so that a coordinate's decode is one table read.
+        const int nL = 2 * Lw + 1;
+        const bool dec_tab = QW == QK_UNIF && utab != nullptr && a.n * nL <= kWorkerTab;
+        if (dec_tab) {
+            for (int idx = threadIdx.x; idx < a.n * nL; idx += kThreads) {
+                const int w = idx / nL;
+                wtab[idx] = __fmul_rn(sc[w], utab[idx - w * nL]);
+            }
+            compute_sync();
+        }
 #pragma unroll 4
         for (int w = 0; w < a.n; ++w) {
             const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
             const float sw = has_scale<QW>() ? sc[w] : 0.0f;
+            const float *dw = wtab + w * nL;
 #pragma unroll
             for (int k = 0; k < kSlots; ++k) {
                 uint32_t c[4];
                 load_codes4_smem(cw, k * kThreads + threadIdx.x, bw, c);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
+                for (int i = 0; i < 4; ++i)
+                    acc[k][i] = __fadd_rn(acc[k][i], dec_tab ? dw[c[i]] : decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
             }
         }
 #pragma unroll
@@ -250,12 +266,13 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
 // compute warps decode, average, re-quantize and write e_s and the broadcast straight to HBM.
 // Used when Q_s scales are per 4096-tile (or absent) and Q_w's are per 4096-tile (or absent).
 template <int MODE, int QW, int QS>
-__global__ void __launch_bounds__(kThreads + 32, MODE == MODE_W ? 2 : 1) server_staged_kernel(const ServerArgs a)
+__global__ void __launch_bounds__(kThreads + 32, 2) server_staged_kernel(const ServerArgs a)
 {
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ TileSmem sm;
     __shared__ float utab[256];
-    __shared__ float ptab[256];  // scaled-sign workers: the average of every sign pattern
+    __shared__ float wtab[kWorkerTab];  // per tile: the average of every sign pattern (scaled-sign
+                                        // workers) or every worker's decoded grid values (uniform)
     const StagePlan &P = a.plan;
     const int S = P.stages;
     uint64_t *full = reinterpret_cast<uint64_t *>(dsm);
@@ -276,6 +293,7 @@ __global__ void __launch_bounds__(kThreads + 32, MODE == MODE_W ? 2 : 1) server_
     const bool use_tab = QW == QK_UNIF && a.qw.bits <= 8;
     if (use_tab)
         for (int i = threadIdx.x; i <= 2 * Lw; i += blockDim.x) utab[i] = __fdiv_rn(static_cast<float>(i - Lw), Lwf);
+    build_qtab<QS>(a.qs, sm.qtab);
     __syncthreads();
 
     if (warp == kWarps) {  // ---------------------------------------------------------- producer
@@ -329,9 +347,9 @@ __global__ void __launch_bounds__(kThreads + 32, MODE == MODE_W ? 2 : 1) server_
         }
         const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
         if ((tile + 1) * kTile <= d)
-            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, ptab, sm);
+            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, sm);
         else
-            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, ptab, sm);
+            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, sm);
     }
 }
 

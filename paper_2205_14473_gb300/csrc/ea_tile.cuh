@@ -12,6 +12,7 @@ struct TileSmem {
     uint32_t redm[kWarps];
     double bcast;
     float bcastf;
+    float qtab[256];  // the uniform grid's fl(i / L) of the tile's own quantizer (build_qtab)
 };
 
 // Slot k of this thread in tile `tile`: coordinates 4q .. 4q+3.  Consecutive threads own
@@ -26,7 +27,7 @@ __device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
 template <int QK, bool FULL, bool BALLOT = true>
 __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
                                              const QParams &q, uint32_t *words, float *resid, int ef,
-                                             uint64_t seed, uint32_t id, uint32_t t)
+                                             uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
 {
     const int bits = code_bits<QK>(q);
     const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
@@ -43,7 +44,7 @@ __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             float dec = 0.0f;
-            c[i] = (FULL || j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec) : 0u;
+            c[i] = (FULL || j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec, qtab) : 0u;
             e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;
         }
         store_codes4<FULL, BALLOT>(words, qs, bits, c, n_words);
@@ -63,7 +64,7 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
                                             TileSmem &sm)
 {
     if constexpr (!has_scale<QK>()) {
-        encode_store<QK, FULL, BALLOT>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t);
+        encode_store<QK, FULL, BALLOT>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t, nullptr);
         return;
     } else {
         const int64_t tile_lo = tile * kTile;
@@ -86,7 +87,9 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
                 s = block_max_all(mx, sm.redm);
             }
             if (threadIdx.x == 0) scales[tile] = s;
-            encode_store<QK, FULL, BALLOT>(u, s, tile, d, q, words, resid, ef, seed, id, t);
+            // sm.qtab was filled by build_qtab before the reduction's barrier
+            encode_store<QK, FULL, BALLOT>(u, s, tile, d, q, words, resid, ef, seed, id, t,
+                                           (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
             return;
         }
         // PASS_STASH

@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(kThreads, 2) worker_kernel(const WorkerArgs a)
 {
     __shared__ TileSmem sm;
     const int64_t tile = blockIdx.x;
+    build_qtab<QK>(a.q, sm.qtab);  // read after the scale reduction's barrier
     if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK, true>(a, tile, sm);
     else worker_tile<MODE, QK, false>(a, tile, sm);
 }
@@ -82,6 +83,9 @@ __global__ void __launch_bounds__(kThreads) finalize_kernel(const FinalizeArgs a
 template <int QK>
 __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
 {
+    __shared__ float qtab_s[256];
+    const float *qtab = build_qtab<QK>(a.q, qtab_s);
+    __syncthreads();
     const int64_t tile = blockIdx.x;
     const int64_t d = a.d;
     const Grouping &G = a.q.grp;
@@ -106,7 +110,7 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
             c[i] = 0u;
             if (j0 + i < d) {
                 const float s = a.scales[group_of(G, j0 + i, hint)];
-                c[i] = encode1<QK>(u[k][i], s, a.q, Lf, L, U[i], dec);
+                c[i] = encode1<QK>(u[k][i], s, a.q, Lf, L, U[i], dec, qtab);
             }
             e[i] = a.ef ? __fsub_rn(u[k][i], dec) : 0.0f;
         }
@@ -119,7 +123,7 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
 // tile are issued first; with 4096-block scales the tile has one scale.
 // HBM traffic per coordinate: 4 B read + 4 B written + b/8 B of code.
 template <int QK, bool FULL>
-__device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile)
+__device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile, const float *qtab)
 {
     const int64_t d = a.d;
     const Grouping &G = a.q.grp;
@@ -147,7 +151,7 @@ __device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile)
             if (FULL || j0 + i < d) {
                 float s = s_tile;
                 if (has_scale<QK>() && !tile_scale) s = __ldg(a.scales + group_of(G, j0 + i, hint));
-                x[k][i] = __fsub_rn(x[k][i], decode1<QK>(c[k][i], s, a.q, Lf, L, nullptr));
+                x[k][i] = __fsub_rn(x[k][i], decode1<QK>(c[k][i], s, a.q, Lf, L, qtab));
             }
         }
         store4<FULL>(a.x, q, d, x[k]);
@@ -157,9 +161,12 @@ __device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile)
 template <int QK>
 __global__ void __launch_bounds__(kThreads) apply_kernel(const ApplyArgs a)
 {
+    __shared__ float qtab_s[256];
+    const float *qtab = build_qtab<QK>(a.q, qtab_s);
+    if (qtab) __syncthreads();
     const int64_t tile = blockIdx.x;
-    if ((tile + 1) * kTile <= a.d) apply_tile<QK, true>(a, tile);
-    else apply_tile<QK, false>(a, tile);
+    if ((tile + 1) * kTile <= a.d) apply_tile<QK, true>(a, tile, qtab);
+    else apply_tile<QK, false>(a, tile, qtab);
 }
 
 __global__ void fill_kernel(float *p, int64_t count, float value)
