@@ -374,6 +374,24 @@ int second_pass(ea_handle *h, const QHost &q, float *buf, uint32_t *words, float
 
 void ea::set_last_error(const char *msg) { g_last_error = msg; }
 
+cudaError_t ea::launch_server(int mode, const ServerArgs &a, cudaStream_t s)
+{
+    if (mode == MODE_W) {
+        switch (a.qs.kind) {
+        case QK_SIGN: return launch_server_for_qs<MODE_W, QK_SIGN>(a, s);
+        case QK_UNIF: return launch_server_for_qs<MODE_W, QK_UNIF>(a, s);
+        case QK_POW2: return launch_server_for_qs<MODE_W, QK_POW2>(a, s);
+        default: return launch_server_for_qs<MODE_W, QK_IDENT>(a, s);
+        }
+    }
+    switch (a.qs.kind) {
+    case QK_SIGN: return launch_server_for_qs<MODE_S, QK_SIGN>(a, s);
+    case QK_UNIF: return launch_server_for_qs<MODE_S, QK_UNIF>(a, s);
+    case QK_POW2: return launch_server_for_qs<MODE_S, QK_POW2>(a, s);
+    default: return launch_server_for_qs<MODE_S, QK_IDENT>(a, s);
+    }
+}
+
 extern "C" {
 
 int ea_workspace_bytes(const ea_config *cfg, size_t *bytes)
@@ -543,7 +561,7 @@ int ea_server_step(ea_handle *h)
     a.status = h->status;
     a.plan = h->splan;
     const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
-    int r = check_cuda(h, W ? launch_server_w(a, h->stream) : launch_server_s(a, h->stream), "server launch");
+    int r = check_cuda(h, launch_server(W ? MODE_W : MODE_S, a, h->stream), "server launch");
     if (r == EA_OK && h->qs.pass == PASS_STASH)
         r = second_pass(h, h->qs, h->es, h->scodes, h->sscales, static_cast<uint32_t>(h->cfg.n));
     if (r != EA_OK) return r;

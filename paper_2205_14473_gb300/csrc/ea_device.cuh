@@ -68,11 +68,13 @@ __device__ __forceinline__ DF df_add(DF a, DF b)
     return {hi, lo};
 }
 
-// Add x to an accumulator whose error terms are collected in acc.lo (Neumaier's form).
+// Add x >= 0 to an accumulator of non-negative terms, its error terms collected in acc.lo.  With
+// a = max(acc.hi, x) >= b = min(acc.hi, x) >= 0, Dekker's Fast2Sum gives s + e = a + b exactly.
 __device__ __forceinline__ void df_accumulate(DF &acc, float x)
 {
-    float s, e;
-    two_sum(acc.hi, x, s, e);
+    const float a = fmaxf(acc.hi, x), b = fminf(acc.hi, x);
+    const float s = __fadd_rn(a, b);
+    const float e = __fsub_rn(b, __fsub_rn(s, a));
     acc.hi = s;
     acc.lo = __fadd_rn(acc.lo, e);
 }
@@ -118,9 +120,15 @@ __device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if (lane == 0) red[warp] = v;
     compute_sync();
-    DF t = red[0];
+    // every warp combines the eight warp totals with the same shuffle tree, then broadcasts lane 0's
+    DF t = lane < kWarps ? red[lane] : DF{0.0f, 0.0f};
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) t = df_add(t, red[w]);
+    for (int o = kWarps / 2; o > 0; o >>= 1) {
+        DF w{__shfl_down_sync(0xffffffffu, t.hi, o), __shfl_down_sync(0xffffffffu, t.lo, o)};
+        t = df_add(t, w);
+    }
+    t.hi = __shfl_sync(0xffffffffu, t.hi, 0);
+    t.lo = __shfl_sync(0xffffffffu, t.lo, 0);
     if (len <= 0) return 0.0f;
     if ((len & (len - 1)) == 0) {  // len <= 4096 here: the factor 2^-k is a normal binary32
         const int k = __ffsll(static_cast<long long>(len)) - 1;
@@ -135,12 +143,10 @@ __device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red)
 __device__ __forceinline__ float block_max_all(float a, uint32_t *red)
 {
     const uint32_t b = __reduce_max_sync(0xffffffffu, __float_as_uint(a));
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = b;
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) red[threadIdx.x >> 5] = b;
     compute_sync();
-    uint32_t m = red[0];
-#pragma unroll
-    for (int w = 1; w < kWarps; ++w) m = max(m, red[w]);
-    return __uint_as_float(m);
+    return __uint_as_float(__reduce_max_sync(0xffffffffu, lane < kWarps ? red[lane] : 0u));
 }
 
 // CTA-wide maximum of non-negative values (exact: compares bit patterns).
@@ -352,6 +358,22 @@ __device__ __forceinline__ uint32_t spread8_by4(uint32_t x)
 // called by all 32 lanes of the warp.  Codes of coordinates >= d are 0 (caller's job).
 // b = 1: one ballot per component; lanes 8g .. 8g+7 fill word (q_lane0 / 8) + g, whose bit
 // 4l + c is component c of lane 8g + l.
+// b in {2, 4, 8}: the slot's 4b bits, shifted to its place in the word and OR-ed across the 8/b
+// lanes that share the word (compile-time width).
+template <int B, bool FULL>
+__device__ __forceinline__ void store_codes4_narrow(uint32_t *__restrict__ words, int64_t q, const uint32_t c[4],
+                                                    int64_t n_words)
+{
+    constexpr int per_word = 8 / B;  // slots per word: 4 (b=2), 2 (b=4), 1 (b=8)
+    uint32_t v = c[0] | (c[1] << B) | (c[2] << (2 * B)) | (c[3] << (3 * B));
+    const int pos = static_cast<int>(q & (per_word - 1));
+    v <<= pos * 4 * B;
+    if (per_word >= 2) v |= __shfl_xor_sync(0xffffffffu, v, 1);
+    if (per_word >= 4) v |= __shfl_xor_sync(0xffffffffu, v, 2);
+    const int64_t wi = (q * B) >> 3;
+    if (pos == 0 && (FULL || wi < n_words)) words[wi] = v;
+}
+
 template <bool FULL = false, bool BALLOT = true>
 __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64_t q, int bits, const uint32_t c[4],
                                              int64_t n_words)
@@ -377,17 +399,12 @@ __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64
             const int64_t wi = ((q - lane) >> 3) + lane;  // q - lane is lane 0's slot
             if (FULL || wi < n_words) words[wi] = w;
         }
-    } else if (bits <= 8) {
-        uint32_t v = 0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) v |= c[i] << (i * bits);
-        const int per_word = 8 / bits;             // slots per word: 4 (b=2), 2 (b=4), 1 (b=8)
-        const int pos = static_cast<int>(q & (per_word - 1));
-        v <<= pos * 4 * bits;
-        if (per_word >= 2) v |= __shfl_xor_sync(0xffffffffu, v, 1);
-        if (per_word >= 4) v |= __shfl_xor_sync(0xffffffffu, v, 2);
-        const int64_t wi = (q * bits) >> 3;
-        if (pos == 0 && (FULL || wi < n_words)) words[wi] = v;
+    } else if (bits == 2) {
+        store_codes4_narrow<2, FULL>(words, q, c, n_words);
+    } else if (bits == 4) {
+        store_codes4_narrow<4, FULL>(words, q, c, n_words);
+    } else if (bits == 8) {
+        store_codes4_narrow<8, FULL>(words, q, c, n_words);
     } else if (bits == 16) {
         if (FULL || 2 * q < n_words)
             reinterpret_cast<uint2 *>(words)[q] = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));

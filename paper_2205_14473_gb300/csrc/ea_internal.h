@@ -133,8 +133,13 @@ struct ApplyArgs {
 };
 
 cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s);
-cudaError_t launch_server_w(const ServerArgs &a, cudaStream_t s);
-cudaError_t launch_server_s(const ServerArgs &a, cudaStream_t s);
+// The server kernel for one placement and broadcast quantizer kind; each (MODE, QS) pair is
+// instantiated only in its own translation unit, ea_server_<mode>_q<QS>.cu.
+template <int MODE, int QS>
+cudaError_t launch_server_for_qs(const ServerArgs &a, cudaStream_t s);
+
+// The server kernel for the placement and the broadcast quantizer kind of `a` (ea_api.cu).
+cudaError_t launch_server(int mode, const ServerArgs &a, cudaStream_t s);
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s);
 cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s);
 cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s);

@@ -150,6 +150,41 @@ __device__ __forceinline__ bool compute_all(bool ok)
     return r != 0;
 }
 
+// Sum, in worker order, the decoded values of n workers' B-bit uniform-grid codes of this thread's
+// four slots, reading each decoded value from the per-tile table wtab (worker w's 2^B - 1 values
+// from w * (2^B - 1)).  The worker loop is unrolled by 8 with a compile-time code width.
+template <int B>
+__device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, uint32_t chunk, int n, const float *wtab,
+                                                float (&acc)[kSlots][4])
+{
+    constexpr int nL = (1 << B) - 1;
+    constexpr uint32_t mask = (1u << B) - 1u;
+    for (int w0 = 0; w0 < n; w0 += 8) {
+#pragma unroll
+        for (int dw = 0; dw < 8; ++dw) {
+            const int w = w0 + dw;
+            if (w < n) {
+                const uint32_t *cw = reinterpret_cast<const uint32_t *>(codes + static_cast<size_t>(w) * chunk);
+                const float *tw = wtab + w * nL;
+#pragma unroll
+                for (int k = 0; k < kSlots; ++k) {
+                    const int ls = k * kThreads + static_cast<int>(threadIdx.x);
+                    const uint32_t word = cw[(ls * B) >> 3];
+                    const int sh = ((ls * B) & 7) * 4;
+                    // the code times 4 (a byte offset into tw) straight from the word: one shift and one mask
+                    const unsigned char *tb = reinterpret_cast<const unsigned char *>(tw);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        // rotating right by (position - 2) mod 32 puts the field at bits 2 .. B+1
+                        const uint32_t off = __funnelshift_r(word, word, (sh + i * B - 2) & 31) & (mask << 2);
+                        acc[k][i] = __fadd_rn(acc[k][i], *reinterpret_cast<const float *>(tb + off));
+                    }
+                }
+            }
+        }
+    }
+}
+
 // One tile of the staged server on the compute warps: the stage `st` holds e_s (m_s, v_s), the
 // workers' code chunks and scales.  The stage is released (arrive on `empty`) as soon as it has
 // been read, before the re-quantization.
@@ -166,7 +201,10 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
     const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
     float acc[kSlots][4];  // the average of the decoded worker messages
     const float *sc = reinterpret_cast<const float *>(st + P.off_scales);
-    if (QW == QK_SIGN && a.n <= 8) {
+    bool done = false;
+    if constexpr (QW == QK_SIGN) {
+      if (a.n <= 8) {
+        done = true;
         // Scaled-sign workers, n <= 8: a coordinate's average depends only on its n sign bits.
         // Thread p forms the worker-order sum for sign pattern p, exactly as the per-coordinate
         // loop would, divides by n, and the coordinates look their average up.  The pattern of
@@ -188,12 +226,19 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
             const int wi = (k * kThreads + static_cast<int>(threadIdx.x)) >> 3;
             uint32_t X = 0;  // bit 4w + i = worker w's code of coordinate i of the slot
 #pragma unroll
-            for (int w = 0; w < 8; ++w)
-                if (w < a.n) X |= ((c0[w * (kTile / 32) + wi] >> sh) & 0xfu) << (4 * w);
+            for (int w = 0; w < 8; ++w) {
+                // rotate worker w's word so that this thread's nibble lands at bits 4w .. 4w+3
+                if (w < a.n) {
+                    const uint32_t word = c0[w * (kTile / 32) + wi];
+                    X |= __funnelshift_r(word, word, (sh - 4 * w) & 31) & (0xfu << (4 * w));
+                }
+            }
 #pragma unroll
             for (int i = 0; i < 4; ++i) acc[k][i] = wtab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
         }
-    } else {
+      }
+    }
+    if (!done) {
 #pragma unroll
         for (int k = 0; k < kSlots; ++k)
 #pragma unroll
@@ -209,18 +254,30 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
             }
             compute_sync();
         }
+        bool summed = false;
+        if constexpr (QW == QK_UNIF) {
+            if (dec_tab && bw == 4) {
+                unif_decode_sum<4>(st + P.off_codes, P.code_chunk, a.n, wtab, acc);
+                summed = true;
+            } else if (dec_tab && bw == 8) {
+                unif_decode_sum<8>(st + P.off_codes, P.code_chunk, a.n, wtab, acc);
+                summed = true;
+            }
+        }
+        if (!summed) {
 #pragma unroll 4
-        for (int w = 0; w < a.n; ++w) {
-            const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
-            const float sw = has_scale<QW>() ? sc[w] : 0.0f;
-            const float *dw = wtab + w * nL;
+            for (int w = 0; w < a.n; ++w) {
+                const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
+                const float sw = has_scale<QW>() ? sc[w] : 0.0f;
+                const float *dw = wtab + w * nL;
 #pragma unroll
-            for (int k = 0; k < kSlots; ++k) {
-                uint32_t c[4];
-                load_codes4_smem(cw, k * kThreads + threadIdx.x, bw, c);
+                for (int k = 0; k < kSlots; ++k) {
+                    uint32_t c[4];
+                    load_codes4_smem(cw, k * kThreads + threadIdx.x, bw, c);
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    acc[k][i] = __fadd_rn(acc[k][i], dec_tab ? dw[c[i]] : decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
+                    for (int i = 0; i < 4; ++i)
+                        acc[k][i] = __fadd_rn(acc[k][i], dec_tab ? dw[c[i]] : decode1<QW>(c[i], sw, a.qw, Lwf, Lw, utab));
+                }
             }
         }
 #pragma unroll
@@ -367,36 +424,31 @@ static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
     return cudaGetLastError();
 }
 
-template <int MODE, int QW>
-static cudaError_t launch_server_qw(const ServerArgs &a, cudaStream_t s)
+// Launch the server kernel for one placement and one broadcast quantizer kind (each (MODE, QS) pair
+// is instantiated in a translation unit of its own, ea_server_<mode>_q<QS>.cu).
+template <int MODE, int QS>
+cudaError_t launch_server_for_qs(const ServerArgs &a, cudaStream_t s)
 {
-    if (a.plan.enabled) {
-        switch (a.qs.kind) {
-        case QK_SIGN: return launch_server_staged<MODE, QW, QK_SIGN>(a, s);
-        case QK_UNIF: return launch_server_staged<MODE, QW, QK_UNIF>(a, s);
-        case QK_POW2: return launch_server_staged<MODE, QW, QK_POW2>(a, s);
-        default: return launch_server_staged<MODE, QW, QK_IDENT>(a, s);
-        }
-    }
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
-    switch (a.qs.kind) {
-    case QK_SIGN: server_kernel<MODE, QW, QK_SIGN><<<grid, block, 0, s>>>(a); break;
-    case QK_UNIF: server_kernel<MODE, QW, QK_UNIF><<<grid, block, 0, s>>>(a); break;
-    case QK_POW2: server_kernel<MODE, QW, QK_POW2><<<grid, block, 0, s>>>(a); break;
-    default: server_kernel<MODE, QW, QK_IDENT><<<grid, block, 0, s>>>(a); break;
+    switch (a.qw.kind) {
+    case QK_SIGN:
+        if (a.plan.enabled) return launch_server_staged<MODE, QK_SIGN, QS>(a, s);
+        server_kernel<MODE, QK_SIGN, QS><<<grid, block, 0, s>>>(a);
+        break;
+    case QK_UNIF:
+        if (a.plan.enabled) return launch_server_staged<MODE, QK_UNIF, QS>(a, s);
+        server_kernel<MODE, QK_UNIF, QS><<<grid, block, 0, s>>>(a);
+        break;
+    case QK_POW2:
+        if (a.plan.enabled) return launch_server_staged<MODE, QK_POW2, QS>(a, s);
+        server_kernel<MODE, QK_POW2, QS><<<grid, block, 0, s>>>(a);
+        break;
+    default:
+        if (a.plan.enabled) return launch_server_staged<MODE, QK_IDENT, QS>(a, s);
+        server_kernel<MODE, QK_IDENT, QS><<<grid, block, 0, s>>>(a);
+        break;
     }
     return cudaGetLastError();
-}
-
-template <int MODE>
-static cudaError_t launch_server_mode(const ServerArgs &a, cudaStream_t s)
-{
-    switch (a.qw.kind) {
-    case QK_SIGN: return launch_server_qw<MODE, QK_SIGN>(a, s);
-    case QK_UNIF: return launch_server_qw<MODE, QK_UNIF>(a, s);
-    case QK_POW2: return launch_server_qw<MODE, QK_POW2>(a, s);
-    default: return launch_server_qw<MODE, QK_IDENT>(a, s);
-    }
 }
 
 }  // namespace ea

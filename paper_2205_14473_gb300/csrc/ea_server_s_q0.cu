@@ -1,0 +1,6 @@
+// ea_server_s_q0.cu -- server kernels, Adam moments at the server, identity broadcast.
+#include "ea_server.cuh"
+
+namespace ea {
+template cudaError_t launch_server_for_qs<MODE_S, QK_IDENT>(const ServerArgs &, cudaStream_t);
+}  // namespace ea

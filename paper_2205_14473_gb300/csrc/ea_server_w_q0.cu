@@ -1,0 +1,6 @@
+// ea_server_w_q0.cu -- server kernels, Adam moments at the workers (the paper's Algorithm 1), identity broadcast.
+#include "ea_server.cuh"
+
+namespace ea {
+template cudaError_t launch_server_for_qs<MODE_W, QK_IDENT>(const ServerArgs &, cudaStream_t);
+}  // namespace ea

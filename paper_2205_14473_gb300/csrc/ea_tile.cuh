@@ -24,11 +24,17 @@ __device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
 
 // Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
 // FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
-template <int QK, bool FULL, bool BALLOT = true>
-__device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
-                                             const QParams &q, uint32_t *words, float *resid, int ef,
-                                             uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
+// Variants of the per-coordinate encode, chosen once per tile: the uniform grid's zero scale
+// (every q = 0), deterministic or stochastic rounding, decode from the fl(i/L) table or by division.
+enum EncVar : int { ENC_PLAIN = 0, ENC_UZERO, ENC_UDET_TAB, ENC_UDET_DIV, ENC_USTO_TAB, ENC_USTO_DIV };
+
+template <int QK, bool FULL, bool BALLOT, int VAR>
+__device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
+                                               const QParams &q, uint32_t *words, float *resid, int ef,
+                                               uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
 {
+    constexpr bool STO = VAR == ENC_USTO_TAB || VAR == ENC_USTO_DIV;
+    constexpr bool TAB = VAR == ENC_UDET_TAB || VAR == ENC_USTO_TAB;
     const int bits = code_bits<QK>(q);
     const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
     const float Lf = static_cast<float>(L);
@@ -38,17 +44,58 @@ __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int
         const int64_t qs = slot_of(tile, k);
         const int64_t j0 = 4 * qs;
         float U[4] = {0.f, 0.f, 0.f, 0.f};
-        if (QK == QK_UNIF && q.stochastic && (FULL || j0 < d)) uniforms4(seed, id, t, j0, U);
+        if (STO && (FULL || j0 < d)) uniforms4(seed, id, t, j0, U);
         uint32_t c[4];
         float e[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             float dec = 0.0f;
-            c[i] = (FULL || j0 + i < d) ? encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec, qtab) : 0u;
+            uint32_t code = 0u;
+            if (VAR == ENC_PLAIN) {
+                code = encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec, qtab);
+            } else if (VAR == ENC_UZERO) {
+                code = static_cast<uint32_t>(L);  // Example 1: Q = 0 when the scale is 0
+            } else {
+                // Example 1 with s > 0: z = u / s, y = z L, then the grid index (see unif_index)
+                const float y = __fmul_rn(__fdiv_rn(u[k][i], s), Lf);
+                int qi;
+                if (STO) {
+                    const float f = floorf(y);
+                    qi = static_cast<int>(f) + (U[i] < __fsub_rn(y, f) ? 1 : 0);
+                } else {
+                    qi = __float2int_rn(y);
+                }
+                dec = __fmul_rn(s, TAB ? qtab[qi + L] : __fdiv_rn(static_cast<float>(qi), Lf));
+                code = static_cast<uint32_t>(qi + L);
+            }
+            c[i] = (FULL || j0 + i < d) ? code : 0u;
             e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;
         }
         store_codes4<FULL, BALLOT>(words, qs, bits, c, n_words);
         if (ef && (FULL || j0 < d)) store4<FULL>(resid, qs, d, e);
+    }
+}
+
+// Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
+// FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
+template <int QK, bool FULL, bool BALLOT = true>
+__device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
+                                             const QParams &q, uint32_t *words, float *resid, int ef,
+                                             uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
+{
+    if constexpr (QK == QK_UNIF) {
+        if (!(s > 0.0f))
+            encode_store_v<QK, FULL, BALLOT, ENC_UZERO>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        else if (q.stochastic && qtab)
+            encode_store_v<QK, FULL, BALLOT, ENC_USTO_TAB>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        else if (q.stochastic)
+            encode_store_v<QK, FULL, BALLOT, ENC_USTO_DIV>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        else if (qtab)
+            encode_store_v<QK, FULL, BALLOT, ENC_UDET_TAB>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        else
+            encode_store_v<QK, FULL, BALLOT, ENC_UDET_DIV>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+    } else {
+        encode_store_v<QK, FULL, BALLOT, ENC_PLAIN>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
     }
 }
 
