@@ -105,37 +105,39 @@ __device__ __forceinline__ double block_sum(DF v, DF *red, double *bcast)
     return r;
 }
 
-// Group scale of the scaled sign, ||u||_1 / G, for a group that is exactly this CTA's tile.  One
-// barrier: every thread combines the eight warp totals in the same order, so all get the same
-// value without a broadcast.  For G a power of two, RN32((hi + lo) / G) = RN32(hi + lo) * 2^-k is
-// one binary32 addition and an exact scaling; other lengths (a ragged last tile) divide in
-// binary64.  The caller must barrier before `red` is reused.
-__device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red)
+// Group scale of the scaled sign, ||u||_1 / G, for a group that is exactly this CTA's tile.
+// Every thread leaves its partial pair in red256; warp 0 combines the 256 pairs (8 per lane in
+// index order, then a 5-level shuffle tree) and broadcasts the scale through *bcastf.  For G a
+// power of two, RN32((hi + lo) / G) = RN32(hi + lo) * 2^-k is one binary32 addition and an exact
+// scaling; other lengths (a ragged last tile) divide in binary64.  Two barriers; red256 and bcastf
+// may be reused after the function returns.
+__device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red256, float *bcastf)
 {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        DF w{__shfl_down_sync(0xffffffffu, v.hi, o), __shfl_down_sync(0xffffffffu, v.lo, o)};
-        v = df_add(v, w);
-    }
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    if (lane == 0) red[warp] = v;
+    red256[threadIdx.x] = v;
     compute_sync();
-    // every warp combines the eight warp totals with the same shuffle tree, then broadcasts lane 0's
-    DF t = lane < kWarps ? red[lane] : DF{0.0f, 0.0f};
+    if (threadIdx.x < 32) {
+        DF t = red256[threadIdx.x];
 #pragma unroll
-    for (int o = kWarps / 2; o > 0; o >>= 1) {
-        DF w{__shfl_down_sync(0xffffffffu, t.hi, o), __shfl_down_sync(0xffffffffu, t.lo, o)};
-        t = df_add(t, w);
+        for (int j = 1; j < kThreads / 32; ++j) t = df_add(t, red256[threadIdx.x + 32 * j]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            DF w{__shfl_down_sync(0xffffffffu, t.hi, o), __shfl_down_sync(0xffffffffu, t.lo, o)};
+            t = df_add(t, w);
+        }
+        if (threadIdx.x == 0) {
+            float s = 0.0f;
+            if (len > 0 && (len & (len - 1)) == 0) {  // len <= 4096 here: 2^-k is a normal binary32
+                const int k = __ffsll(static_cast<long long>(len)) - 1;
+                s = __fmul_rn(__fadd_rn(t.hi, t.lo), __uint_as_float(static_cast<uint32_t>(127 - k) << 23));
+            } else if (len > 0) {
+                const double l1 = static_cast<double>(t.hi) + static_cast<double>(t.lo);
+                s = __double2float_rn(__ddiv_rn(l1, static_cast<double>(len)));
+            }
+            *bcastf = s;
+        }
     }
-    t.hi = __shfl_sync(0xffffffffu, t.hi, 0);
-    t.lo = __shfl_sync(0xffffffffu, t.lo, 0);
-    if (len <= 0) return 0.0f;
-    if ((len & (len - 1)) == 0) {  // len <= 4096 here: the factor 2^-k is a normal binary32
-        const int k = __ffsll(static_cast<long long>(len)) - 1;
-        return __fmul_rn(__fadd_rn(t.hi, t.lo), __uint_as_float(static_cast<uint32_t>(127 - k) << 23));
-    }
-    const double l1 = static_cast<double>(t.hi) + static_cast<double>(t.lo);
-    return __double2float_rn(__ddiv_rn(l1, static_cast<double>(len)));
+    compute_sync();
+    return *bcastf;
 }
 
 // CTA-wide maximum for a group that is exactly this CTA's tile: one barrier, every thread combines

@@ -191,7 +191,7 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, uint
 template <int MODE, int QW, int QS, bool FULL>
 __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
                                                    uint64_t *empty, int Lw, float Lwf, const float *utab,
-                                                   float *wtab, TileSmem &sm)
+                                                   float *wtab, const uint32_t (&flip)[8], TileSmem &sm)
 {
     const StagePlan &P = a.plan;
     const int64_t d = a.d;
@@ -211,11 +211,12 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
         // coordinate i of a slot is gathered from X (bit 4w + i = worker w's code) by one multiply:
         // ((X >> i) & 0x11111111) * 0x01020408 carries no bits and leaves worker w's code at bit
         // 24 + pi(w), pi = (0, 4, 1, 5, 2, 6, 3, 7); the table is indexed in that order.
-        if (threadIdx.x < 256) {
-            constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
+        {
+            // thread p's sign of worker w is bit pi(w) of p: flip[w] holds it as a binary32 sign bit
             float t = 0.0f;
-            for (int w = 0; w < a.n; ++w)
-                t = __fadd_rn(t, ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? sc[w] : -sc[w]);
+#pragma unroll
+            for (int w = 0; w < 8; ++w)
+                if (w < a.n) t = __fadd_rn(t, __uint_as_float(__float_as_uint(sc[w]) ^ flip[w]));
             wtab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
         }
         compute_sync();
@@ -323,7 +324,8 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
 // compute warps decode, average, re-quantize and write e_s and the broadcast straight to HBM.
 // Used when Q_s scales are per 4096-tile (or absent) and Q_w's are per 4096-tile (or absent).
 template <int MODE, int QW, int QS>
-__global__ void __launch_bounds__(kThreads + 32, 2) server_staged_kernel(const ServerArgs a)
+__global__ void __launch_bounds__(kThreads + 32, (MODE == MODE_W && QW == QK_SIGN) ? 3 : 2)
+    server_staged_kernel(const ServerArgs a)
 {
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ TileSmem sm;
@@ -394,6 +396,14 @@ __global__ void __launch_bounds__(kThreads + 32, 2) server_staged_kernel(const S
 
     // ------------------------------------------------------------------------- compute warps
     const int64_t d = a.d;
+    // sign-pattern table (scaled-sign workers): this thread's pattern p = threadIdx.x gives worker w
+    // the sign of bit pi(w) of p, pi = (0, 4, 1, 5, 2, 6, 3, 7); kept as a binary32 sign-bit mask
+    uint32_t flip[8];
+    {
+        constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
+#pragma unroll
+        for (int w = 0; w < 8; ++w) flip[w] = ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? 0u : 0x80000000u;
+    }
     int64_t it = 0;
     for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
         const int s = static_cast<int>(it % S);
@@ -404,9 +414,9 @@ __global__ void __launch_bounds__(kThreads + 32, 2) server_staged_kernel(const S
         }
         const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
         if ((tile + 1) * kTile <= d)
-            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, sm);
+            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
         else
-            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, sm);
+            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
     }
 }
 

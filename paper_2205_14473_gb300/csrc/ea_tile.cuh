@@ -8,6 +8,7 @@
 namespace ea {
 
 struct TileSmem {
+    DF red256[kThreads];  // per-thread partial pairs of the l1 scale
     DF red[kWarps];
     uint32_t redm[kWarps];
     double bcast;
@@ -124,7 +125,7 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
                 for (int k = 0; k < kSlots; ++k)
 #pragma unroll
                     for (int i = 0; i < 4; ++i) df_accumulate(acc, fabsf(u[k][i]));  // invalid u are 0
-                s = block_sign_scale(acc, tile_hi - tile_lo, sm.red);
+                s = block_sign_scale(acc, tile_hi - tile_lo, sm.red256, &sm.bcastf);
             } else {
                 float mx = 0.0f;
 #pragma unroll
