@@ -23,6 +23,32 @@ __device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
     return tile * (kTile / 4) + k * kThreads + threadIdx.x;
 }
 
+// Example 1's grid index of u (|u| <= s, s > 0) without a division.  z = RN(u / s) and y = RN(z L)
+// are stood in for by z' = RN(u r), y' = RN(z' L) with r = RN(1 / s), which the caller computes
+// once per tile.  For s in [2^-125, 2^125] the relative errors of r, z', z and the two products
+// (each at most 2^-24, |z| <= 1) give |y' - y| <= 5.01 * 2^-24 * L, below the margin m = L * 2^-20.
+// The index changes only where y crosses a half-integer (round to nearest even) or, for the
+// stochastic rule, an integer or the draw U; when y' is farther than m from every such point, y
+// lies on the same side of each and gets the same index (so does u = 0, where y' = y = 0).
+// Returns false otherwise, and for r = NaN, which the caller passes for scales outside the range:
+// the caller then takes the index from unif_index, whose division gives z itself.
+template <bool STO>
+__device__ __forceinline__ bool unif_index_fast(float u, float r, float Lf, float m, float U, int &qi)
+{
+    const float y = __fmul_rn(__fmul_rn(u, r), Lf);
+    if constexpr (STO) {
+        const float f = floorf(y);
+        const float fr = __fsub_rn(y, f);  // exact: |y| <= L + 1 < 2^23
+        qi = static_cast<int>(f) + (U < fr ? 1 : 0);
+        // u = 0 gives y' = y = 0 and index 0 exactly
+        return (fr > m && fr < __fsub_rn(1.0f, m) && fabsf(__fsub_rn(U, fr)) > m) || u == 0.0f;
+    } else {
+        const float rn = rintf(y);
+        qi = static_cast<int>(rn);
+        return fabsf(__fsub_rn(y, rn)) < __fsub_rn(0.5f, m);
+    }
+}
+
 // Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
 // FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
 // Variants of the per-coordinate encode, chosen once per tile: the uniform grid's zero scale
@@ -36,10 +62,16 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
 {
     constexpr bool STO = VAR == ENC_USTO_TAB || VAR == ENC_USTO_DIV;
     constexpr bool TAB = VAR == ENC_UDET_TAB || VAR == ENC_USTO_TAB;
+    constexpr bool GRID = VAR != ENC_PLAIN && VAR != ENC_UZERO;
     const int bits = code_bits<QK>(q);
     const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
     const float Lf = static_cast<float>(L);
     const int64_t n_words = (d * bits + 31) >> 5;
+    float r = 0.0f, m = 0.0f;
+    if (GRID) {
+        r = (s >= 0x1p-125f && s <= 0x1p125f) ? __frcp_rn(s) : __int_as_float(0x7fc00000);
+        m = __fmul_rn(Lf, 0x1p-20f);
+    }
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t qs = slot_of(tile, k);
@@ -48,6 +80,18 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
         if (STO && (FULL || j0 < d)) uniforms4(seed, id, t, j0, U);
         uint32_t c[4];
         float e[4];
+        int qi[4] = {0, 0, 0, 0};
+        if (GRID) {
+            // Example 1 with s > 0: the index of y = RN(RN(u / s) L) (see unif_index_fast)
+            bool ok[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) ok[i] = unif_index_fast<STO>(u[k][i], r, Lf, m, U[i], qi[i]);
+            if (!(ok[0] && ok[1] && ok[2] && ok[3])) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    if (!ok[i]) qi[i] = unif_index(u[k][i], s, Lf, STO, U[i]);
+            }
+        }
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             float dec = 0.0f;
@@ -57,17 +101,8 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
             } else if (VAR == ENC_UZERO) {
                 code = static_cast<uint32_t>(L);  // Example 1: Q = 0 when the scale is 0
             } else {
-                // Example 1 with s > 0: z = u / s, y = z L, then the grid index (see unif_index)
-                const float y = __fmul_rn(__fdiv_rn(u[k][i], s), Lf);
-                int qi;
-                if (STO) {
-                    const float f = floorf(y);
-                    qi = static_cast<int>(f) + (U[i] < __fsub_rn(y, f) ? 1 : 0);
-                } else {
-                    qi = __float2int_rn(y);
-                }
-                dec = __fmul_rn(s, TAB ? qtab[qi + L] : __fdiv_rn(static_cast<float>(qi), Lf));
-                code = static_cast<uint32_t>(qi + L);
+                dec = __fmul_rn(s, TAB ? qtab[qi[i] + L] : __fdiv_rn(static_cast<float>(qi[i]), Lf));
+                code = static_cast<uint32_t>(qi[i] + L);
             }
             c[i] = (FULL || j0 + i < d) ? code : 0u;
             e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;

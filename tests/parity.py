@@ -28,6 +28,12 @@ from paper_2205_14473_gb300 import workloads as W
 ATOL, RTOL, SCALE_RTOL = 1e-7, 1e-5, 1e-6
 
 
+def _agree(g: torch.Tensor, w: torch.Tensor, rtol: float, atol: float) -> torch.Tensor:
+    """Within atol + rtol |w|, or equal (infinities of one sign), or NaN on both sides; a NaN or an
+    infinity on one side only disagrees."""
+    return ((g - w).abs() <= atol + rtol * w.abs()) | (g == w) | (g.isnan() & w.isnan())
+
+
 def _offsets(d, spec: W.QuantSpec):
     if spec.kind in (W.Q_IDENTITY, W.Q_POW2):
         return O.group_offsets(d, 0)
@@ -134,9 +140,9 @@ class Lockstep:
         w = self._dev(want).double()
         g = got.double()
         err = (g - w).abs()
-        bad = (err > ATOL + RTOL * w.abs()) & ~self.tainted
+        bad = ~_agree(g, w, RTOL, ATOL) & ~self.tainted
         nbad = int(bad.sum())
-        rel = (err / (w.abs() + 1e-30)).masked_fill(self.tainted, 0)
+        rel = torch.nan_to_num(err / (w.abs() + 1e-30), nan=0.0).masked_fill(self.tainted, 0)
         rep.max_rel[name] = float(rel.max()) if rel.numel() else 0.0
         if nbad:
             j = int(torch.nonzero(bad)[0])
@@ -217,7 +223,7 @@ class Lockstep:
         if bool(self.tainted.any()):
             tainted_groups = np.unique(self._group_ids(offs_full)[self.tainted.cpu().numpy()])
         w = self._dev(want).double()
-        err = (g.double() - w).abs() > SCALE_RTOL * w.abs()
+        err = ~_agree(g.double(), w, SCALE_RTOL, 0.0)
         if len(tainted_groups):
             mask = np.ones(len(want), bool)
             if self.sampled:

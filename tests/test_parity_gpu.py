@@ -81,6 +81,42 @@ def test_quantizer_kinds(qw, qs, gs, placement):
     _run_host(cfg, 4, seed=9, grad_scale=gs)
 
 
+@pytest.mark.parametrize("case,placement", [
+    ("grid_points", ea.ADAM_AT_WORKER), ("grid_points", ea.ADAM_AT_SERVER),
+    ("tiny", ea.ADAM_AT_WORKER), ("tiny", ea.ADAM_AT_SERVER),
+    ("huge", ea.ADAM_AT_WORKER), ("huge", ea.ADAM_AT_SERVER),
+])
+def test_uniform_grid_boundaries_and_scale_range(case, placement):
+    """Example 1's encode away from its common case: inputs on the grid and exact zeros, where
+    y = z L falls on an integer (the stochastic rule's boundary), and group scales below 2^-125
+    (subnormal inputs) or above 2^125, outside the range of the division-free index."""
+    d, n = 10_000, (2 if case == "huge" else 3)
+    alpha = {"grid_points": 1e-3, "tiny": 1e-41, "huge": 1.5e37 if placement == ea.ADAM_AT_WORKER else 1e-3}[case]
+    cfg = ea.EAConfig(d=d, n=n, qw=W.uniform_q(4, 4096, True), qs=W.uniform_q(8, 1000, False), alpha=alpha,
+                      placement=placement, seed=21)
+    L = Lockstep(cfg)
+    rng = np.random.default_rng(23)
+    x_host = np.zeros(d, np.float32)
+    x_dev = torch.zeros(d, device="cuda")
+    for t in range(3):
+        gs = []
+        for _ in range(n):
+            if case == "grid_points":
+                g = (rng.integers(-7, 8, d) / 7.0 * (rng.random(d) < 0.5)).astype(np.float32)
+            elif placement == ea.ADAM_AT_WORKER:  # the step alpha m / sqrt(v) carries alpha's scale
+                g = rng.standard_normal(d).astype(np.float32)
+            else:                                 # the workers quantize g + e itself
+                g = (rng.standard_normal(d) * (1e-41 if case == "tiny" else 2e37)).astype(np.float32)
+            gs.append(g)
+        rep = L.round([torch.from_numpy(g).cuda() for g in gs], gs, x_dev, x_host)
+        assert rep.code_mismatches == 0, f"round {t}: {rep.code_mismatches} codes differ"
+    scales = L.gpu.view(ea.EA_VIEW_SCALES_WORKER, 0)[:3].double().abs()
+    if case == "tiny":
+        assert bool((scales < 2.0 ** -125).all()) and bool((scales > 0).all())
+    elif case == "huge":
+        assert bool((scales > 2.0 ** 125).all()) and bool(torch.isfinite(scales).all())
+
+
 def test_replicas_are_identical_and_protocol():
     cfg = ea.EAConfig(d=10_000, n=2, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-3)
     rnd = ea.EARound(cfg)
