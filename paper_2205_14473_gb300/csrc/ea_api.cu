@@ -298,8 +298,6 @@ StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs,
         P.off_c = off;
         off += 4 * kTile;
     }
-    // Two CTAs per SM when two stages fit 100 KB (106 KB with Adam at the server, whose stages hold
-    // m_s and v_s too); otherwise one CTA per SM with up to 200 KB of stages.
     P.code_chunk = static_cast<uint32_t>(kTile / 8 * qw.bits);
     P.off_codes = off;
     const uint64_t codes = static_cast<uint64_t>(P.code_chunk) * c.n;
@@ -308,17 +306,18 @@ StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs,
     P.off_scales = off;
     off += static_cast<uint32_t>(align_up(4 * static_cast<size_t>(c.n), 16));
     P.stage_bytes = static_cast<uint32_t>(align_up(off, 128));
-    // Scaled-sign workers with Adam at the workers: three CTAs per SM (the kernel is built for it)
-    // when three stages fit 66 KB.
-    const bool three = !server_adam && qw.kind == EA_Q_SIGN_L1 && 3 * P.stage_bytes <= 66 * 1024;
-    const uint32_t two_cta = server_adam ? 106 * 1024 : 100 * 1024;
-    const uint32_t budget = three ? 66 * 1024 : (2 * P.stage_bytes <= two_cta) ? two_cta : 200 * 1024;
-    if (2 * P.stage_bytes > budget) return P;
-    P.stages = std::max(2, std::min(6, static_cast<int>(budget / P.stage_bytes)));
-    const uint32_t bars = static_cast<uint32_t>(align_up(2 * 8 * static_cast<size_t>(P.stages), 128));
-    P.smem_bytes = bars + static_cast<uint32_t>(P.stages) * P.stage_bytes;
-    const uint32_t per_cta = P.smem_bytes + 8 * 1024;  // + static shared memory
-    const int per_sm = (three && 3 * per_cta <= 228 * 1024) ? 3 : (2 * per_cta <= 228 * 1024) ? 2 : 1;
+    // As many resident CTAs per SM as shared memory holds with one stage each (the kernel's
+    // registers allow kServerMaxCtasPerSm), then as many stages per CTA as fit, up to six.  The
+    // full/empty barriers of up to eight stages take the first 128 bytes.
+    int per_sm = 0;
+    for (int ctas = kServerMaxCtasPerSm; ctas >= 1 && per_sm == 0; --ctas) {
+        const uint32_t room = std::min(kSmemPerSm / ctas - kServerStaticSmem - kSmemReservedPerCta, kServerMaxDynSmem);
+        if (room < 128 + P.stage_bytes) continue;
+        per_sm = ctas;
+        P.stages = std::min(6, static_cast<int>((room - 128) / P.stage_bytes));
+    }
+    if (per_sm == 0) return P;
+    P.smem_bytes = 128 + static_cast<uint32_t>(P.stages) * P.stage_bytes;
     P.grid = static_cast<int>(std::min<int64_t>(n_tiles, static_cast<int64_t>(sms) * per_sm));
     P.enabled = 1;
     return P;

@@ -12,6 +12,15 @@ namespace ea {
 constexpr int kThreads = 256;
 constexpr int kSlots = 4;
 constexpr int kTile = kThreads * kSlots * 4;
+// The staged server: CTAs of kThreads compute threads and one producer warp, built for up to three
+// resident CTAs per SM; each holds at most kServerStaticSmem bytes of static shared memory (checked
+// where the kernel is defined) and up to kServerMaxDynSmem of stages.  An SM has kSmemPerSm bytes,
+// of which every resident CTA takes kSmemReservedPerCta for the system.
+constexpr int kServerMaxCtasPerSm = 3;
+constexpr uint32_t kServerStaticSmem = 9 * 1024;
+constexpr uint32_t kServerMaxDynSmem = 200 * 1024;
+constexpr uint32_t kSmemPerSm = 228 * 1024;
+constexpr uint32_t kSmemReservedPerCta = 1024;
 constexpr int kWarps = kThreads / 32;
 
 enum QKind : int { QK_IDENT = 0, QK_SIGN = 1, QK_UNIF = 2, QK_POW2 = 3 };

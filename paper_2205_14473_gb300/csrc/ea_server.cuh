@@ -152,42 +152,47 @@ __device__ __forceinline__ bool compute_all(bool ok)
 
 // Sum, in worker order, the decoded values of n workers' B-bit uniform-grid codes of this thread's
 // four slots, reading each decoded value from the per-tile table wtab (worker w's 2^B - 1 values
-// from w * (2^B - 1)).  The worker loop is unrolled by 8 with a compile-time code width.
+// from w * (2^B - 1)); a tile's chunk holds kTile * B / 8 bytes per worker.  For n <= 8 every
+// worker index is a compile-time constant, so the table and chunk offsets fold into the
+// shared-memory addresses; slots are summed one after the other to keep few values live.
 template <int B>
-__device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, uint32_t chunk, int n, const float *wtab,
+__device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int n, const float *wtab,
                                                 float (&acc)[kSlots][4])
 {
     constexpr int nL = (1 << B) - 1;
+    constexpr int chunk_words = kTile * B / 32;
     constexpr uint32_t mask = (1u << B) - 1u;
-    for (int w0 = 0; w0 < n; w0 += 8) {
+    const uint32_t *c0 = reinterpret_cast<const uint32_t *>(codes);
+    const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
+    // the slot's 4B bits start at bit 4 B ls of the chunk, ls = k * kThreads + threadIdx.x
+    const int sh = ((static_cast<int>(threadIdx.x) * B) & 7) * 4;
+    auto add = [&](int k, int w) {
+        const int ls = k * kThreads + static_cast<int>(threadIdx.x);
+        const uint32_t word = c0[w * chunk_words + ((ls * B) >> 3)];
 #pragma unroll
-        for (int dw = 0; dw < 8; ++dw) {
-            const int w = w0 + dw;
-            if (w < n) {
-                const uint32_t *cw = reinterpret_cast<const uint32_t *>(codes + static_cast<size_t>(w) * chunk);
-                const float *tw = wtab + w * nL;
+        for (int i = 0; i < 4; ++i) {
+            // rotating right by (position - 2) mod 32 puts the field, times 4 (a byte offset into
+            // worker w's table), at bits 2 .. B+1: one shift and one mask
+            const uint32_t off = __funnelshift_r(word, word, (sh + i * B - 2) & 31) & (mask << 2);
+            acc[k][i] = __fadd_rn(acc[k][i], *reinterpret_cast<const float *>(tb + 4 * w * nL + off));
+        }
+    };
 #pragma unroll
-                for (int k = 0; k < kSlots; ++k) {
-                    const int ls = k * kThreads + static_cast<int>(threadIdx.x);
-                    const uint32_t word = cw[(ls * B) >> 3];
-                    const int sh = ((ls * B) & 7) * 4;
-                    // the code times 4 (a byte offset into tw) straight from the word: one shift and one mask
-                    const unsigned char *tb = reinterpret_cast<const unsigned char *>(tw);
+    for (int k = 0; k < kSlots; ++k) {
+        if (n <= 8) {
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        // rotating right by (position - 2) mod 32 puts the field at bits 2 .. B+1
-                        const uint32_t off = __funnelshift_r(word, word, (sh + i * B - 2) & 31) & (mask << 2);
-                        acc[k][i] = __fadd_rn(acc[k][i], *reinterpret_cast<const float *>(tb + off));
-                    }
-                }
-            }
+            for (int w = 0; w < 8; ++w)
+                if (w < n) add(k, w);
+        } else {
+#pragma unroll 2
+            for (int w = 0; w < n; ++w) add(k, w);
         }
     }
 }
 
 // One tile of the staged server on the compute warps: the stage `st` holds e_s (m_s, v_s), the
-// workers' code chunks and scales.  The stage is released (arrive on `empty`) as soon as it has
-// been read, before the re-quantization.
+// workers' code chunks and scales.  The stage's e_s slots then hold u until the re-quantization
+// has read it; the stage is released (arrive on `empty`) after that.
 template <int MODE, int QW, int QS, bool FULL>
 __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
                                                    uint64_t *empty, int Lw, float Lwf, const float *utab,
@@ -202,6 +207,9 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
     float acc[kSlots][4];  // the average of the decoded worker messages
     const float *sc = reinterpret_cast<const float *>(st + P.off_scales);
     bool done = false;
+    // wtab is rebuilt below; the previous tile's reads of it end at its scale reduction's barrier,
+    // which a Q_s without scales does not have
+    if constexpr (!has_scale<QS>() && (QW == QK_SIGN || QW == QK_UNIF)) compute_sync();
     if constexpr (QW == QK_SIGN) {
       if (a.n <= 8) {
         done = true;
@@ -258,15 +266,15 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
         bool summed = false;
         if constexpr (QW == QK_UNIF) {
             if (dec_tab && bw == 4) {
-                unif_decode_sum<4>(st + P.off_codes, P.code_chunk, a.n, wtab, acc);
+                unif_decode_sum<4>(st + P.off_codes, a.n, wtab, acc);
                 summed = true;
             } else if (dec_tab && bw == 8) {
-                unif_decode_sum<8>(st + P.off_codes, P.code_chunk, a.n, wtab, acc);
+                unif_decode_sum<8>(st + P.off_codes, a.n, wtab, acc);
                 summed = true;
             }
         }
-        if (!summed) {
-#pragma unroll 4
+        if (!summed) {  // any worker count and code width; kept rolled (it is not the common case)
+#pragma unroll 1
             for (int w = 0; w < a.n; ++w) {
                 const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
                 const float sw = has_scale<QW>() ? sc[w] : 0.0f;
@@ -286,15 +294,19 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
 #pragma unroll
             for (int i = 0; i < 4; ++i) acc[k][i] = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
     }
-    // e_s (and m_s, v_s) are read from the stage only now, to keep registers for the sums
-    float u[kSlots][4];
+    // e_s (and m_s, v_s) are read from the stage only now, to keep registers for the sums.  Each
+    // slot's u goes back into the stage over its e_s (only this thread reads it again), so that no
+    // register holds u across the scale's reduction.
+    float4 *ubuf = reinterpret_cast<float4 *>(const_cast<unsigned char *>(st) + P.off_a);
+    DF l1{0.0f, 0.0f};
+    float mx = 0.0f;
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int ls = k * kThreads + threadIdx.x;
         const int64_t q = slot_of(tile, k);
         const int64_t j0 = 4 * q;
-        float es[4], ms[4], vs[4];
-        to_arr(reinterpret_cast<const float4 *>(st + P.off_a)[ls], es);
+        float es[4], ms[4], vs[4], u[4];
+        to_arr(ubuf[ls], es);
         if (MODE == MODE_S) {
             to_arr(reinterpret_cast<const float4 *>(st + P.off_b)[ls], ms);
             to_arr(reinterpret_cast<const float4 *>(st + P.off_c)[ls], vs);
@@ -303,18 +315,21 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
         for (int i = 0; i < 4; ++i) {
             float step = acc[k][i];
             if (MODE == MODE_S) step = adam_step(step, ms[i], vs[i], a.hp);
-            u[k][i] = (FULL || j0 + i < d) ? __fadd_rn(step, es[i]) : 0.0f;
+            u[i] = (FULL || j0 + i < d) ? __fadd_rn(step, es[i]) : 0.0f;  // invalid u are 0
+            if constexpr (QS == QK_SIGN) df_accumulate(l1, fabsf(u[i]));
+            else mx = fmaxf(mx, fabsf(u[i]));
         }
+        ubuf[ls] = make_float4(u[0], u[1], u[2], u[3]);
         if (MODE == MODE_S && (FULL || j0 < d)) {
             store4<FULL>(a.ms, q, d, ms);
             store4<FULL>(a.vs, q, d, vs);
         }
     }
-    // the stage is no longer read: hand it back to the producer before the tile's epilogue
+    finish_tile_smem<QS, FULL, false>(ubuf, l1, mx, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.seed,
+                                      static_cast<uint32_t>(a.n), a.t, sm);
+    // the stage is no longer read: hand it back to the producer
     __syncwarp();
     if ((threadIdx.x & 31) == 0) mbar_arrive(empty);
-    finish_tile<QS, FULL, false>(u, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.pass, a.seed,
-                                 static_cast<uint32_t>(a.n), a.t, a.partials, sm);
 }
 
 // The server's round with its inputs staged through shared memory.  Persistent CTAs of 8 compute
@@ -324,10 +339,11 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
 // compute warps decode, average, re-quantize and write e_s and the broadcast straight to HBM.
 // Used when Q_s scales are per 4096-tile (or absent) and Q_w's are per 4096-tile (or absent).
 template <int MODE, int QW, int QS>
-__global__ void __launch_bounds__(kThreads + 32, (MODE == MODE_W && QW == QK_SIGN) ? 3 : 2)
-    server_staged_kernel(const ServerArgs a)
+__global__ void __launch_bounds__(kThreads + 32, kServerMaxCtasPerSm) server_staged_kernel(const ServerArgs a)
 {
     extern __shared__ __align__(128) unsigned char dsm[];
+    static_assert(sizeof(TileSmem) + sizeof(float) * (256 + kWorkerTab) + 128 <= kServerStaticSmem,
+                  "the stage plan's bound on static shared memory");
     __shared__ TileSmem sm;
     __shared__ float utab[256];
     __shared__ float wtab[kWorkerTab];  // per tile: the average of every sign pattern (scaled-sign
@@ -425,8 +441,11 @@ static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
 {
     static bool attr_set = false;
     if (!attr_set) {
-        const cudaError_t e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>,
-                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        cudaError_t e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kServerMaxDynSmem);
+        if (e == cudaSuccess)  // all of the SM's unified L1 / shared memory as shared memory
+            e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>,
+                                     cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }

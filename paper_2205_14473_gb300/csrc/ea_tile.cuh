@@ -23,6 +23,25 @@ __device__ __forceinline__ int64_t slot_of(int64_t tile, int k)
     return tile * (kTile / 4) + k * kThreads + threadIdx.x;
 }
 
+// Where a tile's u comes from: this thread's registers (16 values), or shared memory, one float4 per
+// slot at ls = k * kThreads + threadIdx.x.
+struct URegs {
+    float (*u)[4];
+    __device__ __forceinline__ void get(int k, float (&o)[4]) const
+    {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) o[i] = u[k][i];
+    }
+};
+struct USmem {
+    const float4 *p;
+    __device__ __forceinline__ void get(int k, float (&o)[4]) const
+    {
+        const float4 v = p[k * kThreads + threadIdx.x];
+        o[0] = v.x, o[1] = v.y, o[2] = v.z, o[3] = v.w;
+    }
+};
+
 // Example 1's grid index of u (|u| <= s, s > 0) without a division.  z = RN(u / s) and y = RN(z L)
 // are stood in for by z' = RN(u r), y' = RN(z' L) with r = RN(1 / s), which the caller computes
 // once per tile.  For s in [2^-125, 2^125] the relative errors of r, z', z and the two products
@@ -55,8 +74,8 @@ __device__ __forceinline__ bool unif_index_fast(float u, float r, float Lf, floa
 // (every q = 0), deterministic or stochastic rounding, decode from the fl(i/L) table or by division.
 enum EncVar : int { ENC_PLAIN = 0, ENC_UZERO, ENC_UDET_TAB, ENC_UDET_DIV, ENC_USTO_TAB, ENC_USTO_DIV };
 
-template <int QK, bool FULL, bool BALLOT, int VAR>
-__device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
+template <int QK, bool FULL, bool BALLOT, int VAR, class USrc>
+__device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t tile, int64_t d,
                                                const QParams &q, uint32_t *words, float *resid, int ef,
                                                uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
 {
@@ -78,6 +97,8 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
         const int64_t j0 = 4 * qs;
         float U[4] = {0.f, 0.f, 0.f, 0.f};
         if (STO && (FULL || j0 < d)) uniforms4(seed, id, t, j0, U);
+        float uk[4];
+        src.get(k, uk);
         uint32_t c[4];
         float e[4];
         int qi[4] = {0, 0, 0, 0};
@@ -85,11 +106,11 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
             // Example 1 with s > 0: the index of y = RN(RN(u / s) L) (see unif_index_fast)
             bool ok[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) ok[i] = unif_index_fast<STO>(u[k][i], r, Lf, m, U[i], qi[i]);
+            for (int i = 0; i < 4; ++i) ok[i] = unif_index_fast<STO>(uk[i], r, Lf, m, U[i], qi[i]);
             if (!(ok[0] && ok[1] && ok[2] && ok[3])) {
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
-                    if (!ok[i]) qi[i] = unif_index(u[k][i], s, Lf, STO, U[i]);
+                    if (!ok[i]) qi[i] = unif_index(uk[i], s, Lf, STO, U[i]);
             }
         }
 #pragma unroll
@@ -97,7 +118,7 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
             float dec = 0.0f;
             uint32_t code = 0u;
             if (VAR == ENC_PLAIN) {
-                code = encode1<QK>(u[k][i], s, q, Lf, L, U[i], dec, qtab);
+                code = encode1<QK>(uk[i], s, q, Lf, L, U[i], dec, qtab);
             } else if (VAR == ENC_UZERO) {
                 code = static_cast<uint32_t>(L);  // Example 1: Q = 0 when the scale is 0
             } else {
@@ -105,7 +126,7 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
                 code = static_cast<uint32_t>(qi[i] + L);
             }
             c[i] = (FULL || j0 + i < d) ? code : 0u;
-            e[i] = ef ? __fsub_rn(u[k][i], dec) : 0.0f;
+            e[i] = ef ? __fsub_rn(uk[i], dec) : 0.0f;
         }
         store_codes4<FULL, BALLOT>(words, qs, bits, c, n_words);
         if (ef && (FULL || j0 < d)) store4<FULL>(resid, qs, d, e);
@@ -114,8 +135,8 @@ __device__ __forceinline__ void encode_store_v(float (&u)[kSlots][4], float s, i
 
 // Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
 // FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
-template <int QK, bool FULL, bool BALLOT = true>
-__device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int64_t tile, int64_t d,
+template <int QK, bool FULL, bool BALLOT, class USrc>
+__device__ __forceinline__ void encode_store(const USrc &u, float s, int64_t tile, int64_t d,
                                              const QParams &q, uint32_t *words, float *resid, int ef,
                                              uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
 {
@@ -135,6 +156,27 @@ __device__ __forceinline__ void encode_store(float (&u)[kSlots][4], float s, int
     }
 }
 
+// The tile's end when the tile is one scale group (or Q has no scale) and u sits in shared memory
+// (USmem layout); l1 / mx are this thread's partial sum / maximum of |u| over its valid coordinates.
+template <int QK, bool FULL, bool BALLOT>
+__device__ __forceinline__ void finish_tile_smem(const float4 *ubuf, DF l1, float mx, int64_t tile, int64_t d,
+                                                 const QParams &q, uint32_t *words, float *scales, float *resid,
+                                                 int ef, uint64_t seed, uint32_t id, uint32_t t, TileSmem &sm)
+{
+    float s = 0.0f;
+    if constexpr (has_scale<QK>()) {
+        const int64_t tile_lo = tile * kTile;
+        const int64_t tile_hi = min(tile_lo + static_cast<int64_t>(kTile), d);
+        if constexpr (QK == QK_SIGN)
+            s = block_sign_scale(l1, tile_hi - tile_lo, sm.red256, &sm.bcastf);
+        else
+            s = block_max_all(mx, sm.redm);
+        if (threadIdx.x == 0) scales[tile] = s;
+    }
+    encode_store<QK, FULL, BALLOT>(USmem{ubuf}, s, tile, d, q, words, resid, ef, seed, id, t,
+                                   (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
+}
+
 // The tile's end for a quantizer with scale groups.
 //   PASS_FUSED: the tile is exactly one scale group (blocks of 4096): reduce, encode, store.
 //   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
@@ -147,7 +189,7 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
                                             TileSmem &sm)
 {
     if constexpr (!has_scale<QK>()) {
-        encode_store<QK, FULL, BALLOT>(u, 0.0f, tile, d, q, words, resid, ef, seed, id, t, nullptr);
+        encode_store<QK, FULL, BALLOT>(URegs{u}, 0.0f, tile, d, q, words, resid, ef, seed, id, t, nullptr);
         return;
     } else {
         const int64_t tile_lo = tile * kTile;
@@ -171,7 +213,7 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
             }
             if (threadIdx.x == 0) scales[tile] = s;
             // sm.qtab was filled by build_qtab before the reduction's barrier
-            encode_store<QK, FULL, BALLOT>(u, s, tile, d, q, words, resid, ef, seed, id, t,
+            encode_store<QK, FULL, BALLOT>(URegs{u}, s, tile, d, q, words, resid, ef, seed, id, t,
                                            (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
             return;
         }

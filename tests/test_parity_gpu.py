@@ -117,6 +117,19 @@ def test_uniform_grid_boundaries_and_scale_range(case, placement):
         assert bool((scales > 2.0 ** 125).all()) and bool(torch.isfinite(scales).all())
 
 
+@pytest.mark.parametrize("qw,qs,placement", [
+    (W.uniform_q(4, 4096, True), W.pow2_q(-20, -5, 8), ea.ADAM_AT_WORKER),
+    (W.sign_q(4096), W.identity_q(), ea.ADAM_AT_WORKER),
+    (W.uniform_q(4, 4096, True), W.uniform_q(8, 4096, False), ea.ADAM_AT_SERVER),
+])
+def test_staged_server_several_tiles_per_cta(qw, qs, placement):
+    """d large enough that every persistent server CTA runs several tiles through its ring of
+    stages (the per-tile decode tables are rebuilt between tiles), with a ragged last tile."""
+    d = 4096 * 152 * 3 * 2 + 777
+    cfg = ea.EAConfig(d=d, n=3, qw=qw, qs=qs, alpha=1e-3, placement=placement, seed=31)
+    _run_host(cfg, 2, seed=37, grad_scale=1e-3)
+
+
 def test_replicas_are_identical_and_protocol():
     cfg = ea.EAConfig(d=10_000, n=2, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-3)
     rnd = ea.EARound(cfg)
