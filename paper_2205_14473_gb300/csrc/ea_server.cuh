@@ -94,7 +94,7 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
             store4(a.vs, q, d, vs[k]);
         }
     }
-    finish_tile<QS>(u, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.pass, a.seed,
+    finish_tile<QS>(URegs{u}, tile, d, a.qs, a.words, a.scales, a.es, a.ef, a.pass, a.seed,
                     static_cast<uint32_t>(a.n), a.t, a.partials, sm);
 }
 

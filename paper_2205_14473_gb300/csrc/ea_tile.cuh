@@ -177,19 +177,19 @@ __device__ __forceinline__ void finish_tile_smem(const float4 *ubuf, DF l1, floa
                                    (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
 }
 
-// The tile's end for a quantizer with scale groups.
+// The tile's end for a quantizer with scale groups, u read through `src` (URegs or USmem).
 //   PASS_FUSED: the tile is exactly one scale group (blocks of 4096): reduce, encode, store.
 //   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
 // BALLOT: pack 1-bit codes with __ballot_sync (worker kernels) or with shuffles (the server, whose
 // tile loop is instruction-bound).
-template <int QK, bool FULL = false, bool BALLOT = true>
-__device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile, int64_t d, const QParams &q,
+template <int QK, bool FULL = false, bool BALLOT = true, class USrc>
+__device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64_t d, const QParams &q,
                                             uint32_t *words, float *scales, float *resid, int ef, int pass,
                                             uint64_t seed, uint32_t id, uint32_t t, double *partials,
                                             TileSmem &sm)
 {
     if constexpr (!has_scale<QK>()) {
-        encode_store<QK, FULL, BALLOT>(URegs{u}, 0.0f, tile, d, q, words, resid, ef, seed, id, t, nullptr);
+        encode_store<QK, FULL, BALLOT>(src, 0.0f, tile, d, q, words, resid, ef, seed, id, t, nullptr);
         return;
     } else {
         const int64_t tile_lo = tile * kTile;
@@ -199,21 +199,27 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
             if constexpr (QK == QK_SIGN) {
                 DF acc{0.0f, 0.0f};
 #pragma unroll
-                for (int k = 0; k < kSlots; ++k)
+                for (int k = 0; k < kSlots; ++k) {
+                    float uk[4];
+                    src.get(k, uk);
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) df_accumulate(acc, fabsf(u[k][i]));  // invalid u are 0
+                    for (int i = 0; i < 4; ++i) df_accumulate(acc, fabsf(uk[i]));  // invalid u are 0
+                }
                 s = block_sign_scale(acc, tile_hi - tile_lo, sm.red256, &sm.bcastf);
             } else {
                 float mx = 0.0f;
 #pragma unroll
-                for (int k = 0; k < kSlots; ++k)
+                for (int k = 0; k < kSlots; ++k) {
+                    float uk[4];
+                    src.get(k, uk);
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) mx = fmaxf(mx, fabsf(u[k][i]));
+                    for (int i = 0; i < 4; ++i) mx = fmaxf(mx, fabsf(uk[i]));
+                }
                 s = block_max_all(mx, sm.redm);
             }
             if (threadIdx.x == 0) scales[tile] = s;
             // sm.qtab was filled by build_qtab before the reduction's barrier
-            encode_store<QK, FULL, BALLOT>(URegs{u}, s, tile, d, q, words, resid, ef, seed, id, t,
+            encode_store<QK, FULL, BALLOT>(src, s, tile, d, q, words, resid, ef, seed, id, t,
                                            (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
             return;
         }
@@ -221,7 +227,9 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
             const int64_t qs = slot_of(tile, k);
-            if (FULL || 4 * qs < d) store4<FULL>(resid, qs, d, u[k]);
+            float uk[4];
+            src.get(k, uk);
+            if (FULL || 4 * qs < d) store4<FULL>(resid, qs, d, uk);
         }
         const Grouping &G = q.grp;
         for (int64_t gi = first_group_of_tile(G, tile);; ++gi) {
@@ -233,9 +241,11 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
 #pragma unroll
                 for (int k = 0; k < kSlots; ++k) {
                     const int64_t j0 = 4 * slot_of(tile, k);
+                    float uk[4];
+                    src.get(k, uk);
 #pragma unroll
                     for (int i = 0; i < 4; ++i)
-                        if (j0 + i >= lo && j0 + i < hi) df_accumulate(acc, fabsf(u[k][i]));
+                        if (j0 + i >= lo && j0 + i < hi) df_accumulate(acc, fabsf(uk[i]));
                 }
                 part = block_sum(acc, sm.red, &sm.bcast);
             } else {
@@ -243,9 +253,11 @@ __device__ __forceinline__ void finish_tile(float (&u)[kSlots][4], int64_t tile,
 #pragma unroll
                 for (int k = 0; k < kSlots; ++k) {
                     const int64_t j0 = 4 * slot_of(tile, k);
+                    float uk[4];
+                    src.get(k, uk);
 #pragma unroll
                     for (int i = 0; i < 4; ++i)
-                        if (j0 + i >= lo && j0 + i < hi) mx = fmaxf(mx, fabsf(u[k][i]));
+                        if (j0 + i >= lo && j0 + i < hi) mx = fmaxf(mx, fabsf(uk[i]));
                 }
                 part = static_cast<double>(block_max(mx, sm.redm, &sm.bcastf));
             }

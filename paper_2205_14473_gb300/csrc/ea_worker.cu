@@ -4,8 +4,10 @@
 namespace ea {
 
 // One tile of worker_kernel; FULL: the tile lies inside [0, d) (every tile but a ragged last one).
+// Each slot's u goes to ubuf (only this thread reads it again), so that no register holds u across
+// the scale's reduction and more CTAs fit on an SM.
 template <int MODE, int QK, bool FULL>
-__device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, TileSmem &sm)
+__device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, float4 *ubuf, TileSmem &sm)
 {
     const int64_t d = a.d;
     float g[kSlots][4], e[kSlots][4], m[kSlots][4], v[kSlots][4];
@@ -19,37 +21,42 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, T
             load4<FULL>(a.v, q, d, v[k]);
         }
     }
-    float u[kSlots][4];
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t q = slot_of(tile, k);
         const int64_t j0 = 4 * q;
+        float u[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             float step = g[k][i];
             if (MODE == MODE_W) step = adam_step(g[k][i], m[k][i], v[k][i], a.hp);
-            u[k][i] = (FULL || j0 + i < d) ? __fadd_rn(step, e[k][i]) : 0.0f;
+            u[i] = (FULL || j0 + i < d) ? __fadd_rn(step, e[k][i]) : 0.0f;
         }
+        ubuf[k * kThreads + threadIdx.x] = make_float4(u[0], u[1], u[2], u[3]);
         if (MODE == MODE_W && (FULL || j0 < d)) {
             store4<FULL>(a.m, q, d, m[k]);
             store4<FULL>(a.v, q, d, v[k]);
         }
     }
-    finish_tile<QK, FULL>(u, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t, a.partials, sm);
+    finish_tile<QK, FULL>(USmem{ubuf}, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t,
+                          a.partials, sm);
 }
 
 // Algorithm 2 for one worker on one 4096-coordinate tile.  With Adam at the worker:
 //   v <- beta2 v + (1-beta2) g^2, m <- beta1 m + (1-beta1) g, u = alpha m / sqrt(v) + e;
 // with Adam at the server: u = g + e.  Then Q_w(u) and e <- u - Q_w(u) (finish_tile).
 // HBM traffic per coordinate: 16 B read + 12 B written + b/8 B of code (Adam at the worker).
+// Resident CTAs per SM the registers are sized for: four with Adam at the server (g and e per
+// coordinate), three with Adam at the worker, two for its uniform grid (stochastic rounding's draws).
 template <int MODE, int QK>
-__global__ void __launch_bounds__(kThreads, 2) worker_kernel(const WorkerArgs a)
+__global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : (QK == QK_UNIF ? 2 : 3)) worker_kernel(const WorkerArgs a)
 {
     __shared__ TileSmem sm;
+    __shared__ float4 ubuf[kSlots * kThreads];
     const int64_t tile = blockIdx.x;
     build_qtab<QK>(a.q, sm.qtab);  // read after the scale reduction's barrier
-    if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK, true>(a, tile, sm);
-    else worker_tile<MODE, QK, false>(a, tile, sm);
+    if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK, true>(a, tile, ubuf, sm);
+    else worker_tile<MODE, QK, false>(a, tile, ubuf, sm);
 }
 
 // Second pass, one CTA per scale group: combine the group's per-tile partial norms in a fixed
