@@ -152,9 +152,9 @@ __device__ __forceinline__ bool compute_all(bool ok)
 
 // Sum, in worker order, the decoded values of n workers' B-bit uniform-grid codes of this thread's
 // four slots, reading each decoded value from the per-tile table wtab (worker w's 2^B - 1 values
-// from w * (2^B - 1)); a tile's chunk holds kTile * B / 8 bytes per worker.  For n <= 8 every
-// worker index is a compile-time constant, so the table and chunk offsets fold into the
-// shared-memory addresses; slots are summed one after the other to keep few values live.
+// from w * (2^B - 1)); a tile's chunk holds kTile * B / 8 bytes per worker.  The worker loop is
+// kept rolled (two workers per iteration) so that the hot loop stays small in the instruction
+// cache; the slots and coordinates inside it are unrolled.
 template <int B>
 __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int n, const float *wtab,
                                                 float (&acc)[kSlots][4])
@@ -162,30 +162,22 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
     constexpr int nL = (1 << B) - 1;
     constexpr int chunk_words = kTile * B / 32;
     constexpr uint32_t mask = (1u << B) - 1u;
-    const uint32_t *c0 = reinterpret_cast<const uint32_t *>(codes);
-    const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
     // the slot's 4B bits start at bit 4 B ls of the chunk, ls = k * kThreads + threadIdx.x
     const int sh = ((static_cast<int>(threadIdx.x) * B) & 7) * 4;
-    auto add = [&](int k, int w) {
-        const int ls = k * kThreads + static_cast<int>(threadIdx.x);
-        const uint32_t word = c0[w * chunk_words + ((ls * B) >> 3)];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            // rotating right by (position - 2) mod 32 puts the field, times 4 (a byte offset into
-            // worker w's table), at bits 2 .. B+1: one shift and one mask
-            const uint32_t off = __funnelshift_r(word, word, (sh + i * B - 2) & 31) & (mask << 2);
-            acc[k][i] = __fadd_rn(acc[k][i], *reinterpret_cast<const float *>(tb + 4 * w * nL + off));
-        }
-    };
-#pragma unroll
-    for (int k = 0; k < kSlots; ++k) {
-        if (n <= 8) {
-#pragma unroll
-            for (int w = 0; w < 8; ++w)
-                if (w < n) add(k, w);
-        } else {
+    const uint32_t *cw = reinterpret_cast<const uint32_t *>(codes) + ((static_cast<int>(threadIdx.x) * B) >> 3);
+    const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
 #pragma unroll 2
-            for (int w = 0; w < n; ++w) add(k, w);
+    for (int w = 0; w < n; ++w, cw += chunk_words, tb += 4 * nL) {
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            const uint32_t word = cw[(k * kThreads * B) >> 3];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                // rotating right by (position - 2) mod 32 puts the field, times 4 (a byte offset
+                // into worker w's table), at bits 2 .. B+1: one shift and one mask
+                const uint32_t off = __funnelshift_r(word, word, (sh + i * B - 2) & 31) & (mask << 2);
+                acc[k][i] = __fadd_rn(acc[k][i], *reinterpret_cast<const float *>(tb + off));
+            }
         }
     }
 }
