@@ -106,8 +106,8 @@ __device__ __forceinline__ double block_sum(DF v, DF *red, double *bcast)
 }
 
 // Group scale of the scaled sign, ||u||_1 / G, for a group that is exactly this CTA's tile.
-// Every thread leaves its partial pair in red256; warp 0 combines the 256 pairs (8 per lane in
-// index order, then a 5-level shuffle tree) and broadcasts the scale through *bcastf.  For G a
+// Every thread leaves its partial pair in red256; warp 0 combines the 256 pairs (8 per lane in a
+// tree, then a 5-level shuffle tree) and broadcasts the scale through *bcastf.  For G a
 // power of two, RN32((hi + lo) / G) = RN32(hi + lo) * 2^-k is one binary32 addition and an exact
 // scaling; other lengths (a ragged last tile) divide in binary64.  Two barriers; red256 and bcastf
 // may be reused after the function returns.
@@ -116,9 +116,13 @@ __device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red256,
     red256[threadIdx.x] = v;
     compute_sync();
     if (threadIdx.x < 32) {
-        DF t = red256[threadIdx.x];
+        static_assert(kThreads == 256, "eight partials per lane");
+        DF p[8];
 #pragma unroll
-        for (int j = 1; j < kThreads / 32; ++j) t = df_add(t, red256[threadIdx.x + 32 * j]);
+        for (int j = 0; j < 8; ++j) p[j] = red256[threadIdx.x + 32 * j];
+        // a tree of depth 3 over the lane's eight partials, then five shuffle levels: eight
+        // dependent additions in all
+        DF t = df_add(df_add(df_add(p[0], p[1]), df_add(p[2], p[3])), df_add(df_add(p[4], p[5]), df_add(p[6], p[7])));
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             DF w{__shfl_down_sync(0xffffffffu, t.hi, o), __shfl_down_sync(0xffffffffu, t.lo, o)};

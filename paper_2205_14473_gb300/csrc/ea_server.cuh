@@ -186,8 +186,8 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
 // workers' code chunks and scales.  The stage's e_s slots then hold u until the re-quantization
 // has read it; the stage is released (arrive on `empty`) after that.
 template <int MODE, int QW, int QS, bool FULL>
-__device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
-                                                   uint64_t *empty, int Lw, float Lwf, const float *utab,
+__device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
+                                                   bool ok, uint64_t *empty, int Lw, float Lwf, const float *utab,
                                                    float *wtab, const uint32_t (&flip)[8], TileSmem &sm)
 {
     const StagePlan &P = a.plan;
@@ -219,7 +219,9 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
                 if (w < a.n) t = __fadd_rn(t, __uint_as_float(__float_as_uint(sc[w]) ^ flip[w]));
             wtab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
         }
-        compute_sync();
+        // the table's barrier, and agreement on the stage wait: if any thread's wait ran out, the
+        // entries just written may hold stale stage data and the tile is abandoned unread
+        if (!compute_all(ok)) return false;
         const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
         const uint32_t *c0 = reinterpret_cast<const uint32_t *>(st + P.off_codes);
 #pragma unroll
@@ -253,8 +255,8 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
                 const int w = idx / nL;
                 wtab[idx] = __fmul_rn(sc[w], utab[idx - w * nL]);
             }
-            compute_sync();
         }
+        if (!compute_all(ok)) return false;  // the table's barrier and agreement on the stage wait
         bool summed = false;
         if constexpr (QW == QK_UNIF) {
             if (dec_tab && bw == 4) {
@@ -322,6 +324,7 @@ __device__ __forceinline__ void server_staged_tile(const ServerArgs &a, int64_t 
     // the stage is no longer read: hand it back to the producer
     __syncwarp();
     if ((threadIdx.x & 31) == 0) mbar_arrive(empty);
+    return true;
 }
 
 // The server's round with its inputs staged through shared memory.  Persistent CTAs of 8 compute
@@ -415,16 +418,16 @@ __global__ void __launch_bounds__(kThreads + 32, kServerMaxCtasPerSm) server_sta
     int64_t it = 0;
     for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
         const int s = static_cast<int>(it % S);
-        const bool ok = compute_all(mbar_wait(&full[s], static_cast<uint32_t>((it / S) & 1)));
-        if (!ok) {
+        // bounded wait; the tile's first barrier makes every compute thread agree on the outcome
+        const bool ok = mbar_wait(&full[s], static_cast<uint32_t>((it / S) & 1));
+        const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
+        const bool go = (tile + 1) * kTile <= d
+            ? server_staged_tile<MODE, QW, QS, true>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm)
+            : server_staged_tile<MODE, QW, QS, false>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
+        if (!go) {
             if (threadIdx.x == 0) report_status(a.status, kStatusTimeout);
             break;
         }
-        const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
-        if ((tile + 1) * kTile <= d)
-            server_staged_tile<MODE, QW, QS, true>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
-        else
-            server_staged_tile<MODE, QW, QS, false>(a, tile, st, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
     }
 }
 
