@@ -152,14 +152,13 @@ __device__ __forceinline__ bool compute_all(bool ok)
 
 // Sum, in worker order, the decoded values of n workers' B-bit uniform-grid codes of this thread's
 // four slots, reading each decoded value from the per-tile table wtab (worker w's 2^B - 1 values
-// from w * (2^B - 1)); a tile's chunk holds kTile * B / 8 bytes per worker.  The worker loop is
+// from w * 2^B); a tile's chunk holds kTile * B / 8 bytes per worker.  The worker loop is
 // kept rolled (two workers per iteration) so that the hot loop stays small in the instruction
 // cache; the slots and coordinates inside it are unrolled.
 template <int B>
 __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int n, const float *wtab,
                                                 float (&acc)[kSlots][4])
 {
-    constexpr int nL = (1 << B) - 1;
     constexpr int chunk_words = kTile * B / 32;
     constexpr uint32_t mask = (1u << B) - 1u;
     // the slot's 4B bits start at bit 4 B ls of the chunk, ls = k * kThreads + threadIdx.x
@@ -167,7 +166,7 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
     const uint32_t *cw = reinterpret_cast<const uint32_t *>(codes) + ((static_cast<int>(threadIdx.x) * B) >> 3);
     const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
 #pragma unroll 2
-    for (int w = 0; w < n; ++w, cw += chunk_words, tb += 4 * nL) {
+    for (int w = 0; w < n; ++w, cw += chunk_words, tb += 4 << B) {
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
             const uint32_t word = cw[(k * kThreads * B) >> 3];
@@ -248,12 +247,13 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
             for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
         // Uniform-grid workers: every worker's 2L+1 decoded values s_w * fl(i/L) for this tile, as
         // decode1 would form them, so that a coordinate's decode is one table read.
+        // Worker w's table starts at w * 2^b; entries 0 .. 2L = 2^b - 2 are used.
         const int nL = 2 * Lw + 1;
-        const bool dec_tab = QW == QK_UNIF && utab != nullptr && a.n * nL <= kWorkerTab;
+        const bool dec_tab = QW == QK_UNIF && utab != nullptr && (a.n << bw) <= kWorkerTab;
         if (dec_tab) {
-            for (int idx = threadIdx.x; idx < a.n * nL; idx += kThreads) {
-                const int w = idx / nL;
-                wtab[idx] = __fmul_rn(sc[w], utab[idx - w * nL]);
+            for (int idx = threadIdx.x; idx < (a.n << bw); idx += kThreads) {
+                const int i = idx & ((1 << bw) - 1);
+                if (i < nL) wtab[idx] = __fmul_rn(sc[idx >> bw], utab[i]);
             }
         }
         if (!compute_all(ok)) return false;  // the table's barrier and agreement on the stage wait
@@ -272,7 +272,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
             for (int w = 0; w < a.n; ++w) {
                 const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
                 const float sw = has_scale<QW>() ? sc[w] : 0.0f;
-                const float *dw = wtab + w * nL;
+                const float *dw = wtab + (w << bw);
 #pragma unroll
                 for (int k = 0; k < kSlots; ++k) {
                     uint32_t c[4];
@@ -283,10 +283,18 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
                 }
             }
         }
+        // the average: a multiplication by 1/n is exact for n a power of two (one branch per tile)
+        if (pow2n) {
 #pragma unroll
-        for (int k = 0; k < kSlots; ++k)
+            for (int k = 0; k < kSlots; ++k)
 #pragma unroll
-            for (int i = 0; i < 4; ++i) acc[k][i] = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
+                for (int i = 0; i < 4; ++i) acc[k][i] = __fmul_rn(acc[k][i], inv_n);
+        } else {
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[k][i] = __fdiv_rn(acc[k][i], nf);
+        }
     }
     // e_s (and m_s, v_s) are read from the stage only now, to keep registers for the sums.  Each
     // slot's u goes back into the stage over its e_s (only this thread reads it again), so that no
