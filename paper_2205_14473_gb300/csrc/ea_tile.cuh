@@ -74,7 +74,8 @@ __device__ __forceinline__ bool unif_index_fast(float u, float r, float Lf, floa
 // (every q = 0), deterministic or stochastic rounding, decode from the fl(i/L) table or by division.
 enum EncVar : int { ENC_PLAIN = 0, ENC_UZERO, ENC_UDET_TAB, ENC_UDET_DIV, ENC_USTO_TAB, ENC_USTO_DIV };
 
-template <int QK, bool FULL, bool BALLOT, int VAR, class USrc>
+// BITS: the code width as a compile-time constant (0: code_bits of the kind, or q.bits).
+template <int QK, bool FULL, bool BALLOT, int VAR, int BITS, class USrc>
 __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t tile, int64_t d,
                                                const QParams &q, uint32_t *words, float *resid, int ef,
                                                uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
@@ -82,7 +83,7 @@ __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t
     constexpr bool STO = VAR == ENC_USTO_TAB || VAR == ENC_USTO_DIV;
     constexpr bool TAB = VAR == ENC_UDET_TAB || VAR == ENC_USTO_TAB;
     constexpr bool GRID = VAR != ENC_PLAIN && VAR != ENC_UZERO;
-    const int bits = code_bits<QK>(q);
+    const int bits = BITS ? BITS : code_bits<QK>(q);
     const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
     const float Lf = static_cast<float>(L);
     const int64_t n_words = (d * bits + 31) >> 5;
@@ -135,24 +136,44 @@ __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t
 
 // Encode u (valid coordinates only) with scale s, store codes (all lanes) and the residual.
 // FULL: the whole tile lies inside [0, d), so no coordinate needs a bounds check.
+// Example 1 with a compile-time width: for b <= 8 the caller passes qtab (fl(i/L) of the tile's
+// quantizer) and the decode is a table read; 16-bit grids divide.
+template <int QK, bool FULL, bool BALLOT, int BITS, class USrc>
+__device__ __forceinline__ void encode_store_unif(const USrc &u, float s, int64_t tile, int64_t d,
+                                                  const QParams &q, uint32_t *words, float *resid, int ef,
+                                                  uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
+{
+    constexpr bool tab = BITS <= 8;
+    if (!(s > 0.0f))
+        encode_store_v<QK, FULL, BALLOT, ENC_UZERO, BITS>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+    else if (q.stochastic)
+        encode_store_v<QK, FULL, BALLOT, tab ? ENC_USTO_TAB : ENC_USTO_DIV, BITS>(u, s, tile, d, q, words, resid, ef,
+                                                                               seed, id, t, qtab);
+    else
+        encode_store_v<QK, FULL, BALLOT, tab ? ENC_UDET_TAB : ENC_UDET_DIV, BITS>(u, s, tile, d, q, words, resid, ef,
+                                                                               seed, id, t, qtab);
+}
+
+// Encode and store a tile; the variant (and a configured code width) is chosen once per tile.
 template <int QK, bool FULL, bool BALLOT, class USrc>
 __device__ __forceinline__ void encode_store(const USrc &u, float s, int64_t tile, int64_t d,
                                              const QParams &q, uint32_t *words, float *resid, int ef,
                                              uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
 {
     if constexpr (QK == QK_UNIF) {
-        if (!(s > 0.0f))
-            encode_store_v<QK, FULL, BALLOT, ENC_UZERO>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
-        else if (q.stochastic && qtab)
-            encode_store_v<QK, FULL, BALLOT, ENC_USTO_TAB>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
-        else if (q.stochastic)
-            encode_store_v<QK, FULL, BALLOT, ENC_USTO_DIV>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
-        else if (qtab)
-            encode_store_v<QK, FULL, BALLOT, ENC_UDET_TAB>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        switch (q.bits) {  // the widths ea_init accepts
+        case 2: encode_store_unif<QK, FULL, BALLOT, 2>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
+        case 4: encode_store_unif<QK, FULL, BALLOT, 4>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
+        case 8: encode_store_unif<QK, FULL, BALLOT, 8>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
+        default: encode_store_unif<QK, FULL, BALLOT, 16>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
+        }
+    } else if constexpr (QK == QK_POW2) {
+        if (q.bits == 4)
+            encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 4>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
         else
-            encode_store_v<QK, FULL, BALLOT, ENC_UDET_DIV>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+            encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 8>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
     } else {
-        encode_store_v<QK, FULL, BALLOT, ENC_PLAIN>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 0>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
     }
 }
 
