@@ -307,10 +307,12 @@ StagePlan make_server_plan(const ea_config &c, const QHost &qw, const QHost &qs,
     off += static_cast<uint32_t>(align_up(4 * static_cast<size_t>(c.n), 16));
     P.stage_bytes = static_cast<uint32_t>(align_up(off, 128));
     // As many resident CTAs per SM as shared memory holds with one stage each (the kernel's
-    // registers allow kServerMaxCtasPerSm), then as many stages per CTA as fit, up to six.  The
-    // full/empty barriers of up to eight stages take the first 128 bytes.
+    // registers allow server_ctas_per_sm; the EA_Q_* kinds are the kernels' QK_* values), then as
+    // many stages per CTA as fit, up to six.  The full/empty barriers of up to eight stages take
+    // the first 128 bytes.
+    const int max_ctas = server_ctas_per_sm(server_adam ? MODE_S : MODE_W, qw.kind, qs.kind);
     int per_sm = 0;
-    for (int ctas = kServerMaxCtasPerSm; ctas >= 1 && per_sm == 0; --ctas) {
+    for (int ctas = max_ctas; ctas >= 1 && per_sm == 0; --ctas) {
         const uint32_t room = std::min(kSmemPerSm / ctas - kServerStaticSmem - kSmemReservedPerCta, kServerMaxDynSmem);
         if (room < 128 + P.stage_bytes) continue;
         per_sm = ctas;

@@ -12,11 +12,10 @@ namespace ea {
 constexpr int kThreads = 256;
 constexpr int kSlots = 4;
 constexpr int kTile = kThreads * kSlots * 4;
-// The staged server: CTAs of kThreads compute threads and one producer warp, built for up to three
-// resident CTAs per SM; each holds at most kServerStaticSmem bytes of static shared memory (checked
-// where the kernel is defined) and up to kServerMaxDynSmem of stages.  An SM has kSmemPerSm bytes,
-// of which every resident CTA takes kSmemReservedPerCta for the system.
-constexpr int kServerMaxCtasPerSm = 3;
+// The staged server: CTAs of kThreads compute threads and one producer warp, built for up to
+// server_ctas_per_sm resident CTAs per SM; each holds at most kServerStaticSmem bytes of static
+// shared memory (checked where the kernel is defined) and up to kServerMaxDynSmem of stages.  An
+// SM has kSmemPerSm bytes, of which every resident CTA takes kSmemReservedPerCta for the system.
 constexpr uint32_t kServerStaticSmem = 9 * 1024;
 constexpr uint32_t kServerMaxDynSmem = 200 * 1024;
 constexpr uint32_t kSmemPerSm = 228 * 1024;
@@ -26,6 +25,14 @@ constexpr int kWarps = kThreads / 32;
 enum QKind : int { QK_IDENT = 0, QK_SIGN = 1, QK_UNIF = 2, QK_POW2 = 3 };
 enum GKind : int { GK_WHOLE = 0, GK_BLOCK = 1, GK_SEG = 2 };
 enum Mode : int { MODE_W = 0, MODE_S = 1 };  // Adam at the workers (the paper) / at the server
+
+// Resident CTAs per SM a staged server kernel's registers are sized for (its __launch_bounds__, and
+// the stage plan's limit): four (56 registers) for scaled-sign workers and broadcast with Adam at
+// the workers, whose tile needs the fewest live values; three (72 registers) otherwise.
+constexpr int server_ctas_per_sm(int mode, int qw, int qs)
+{
+    return (mode == MODE_W && qw == QK_SIGN && qs == QK_SIGN) ? 4 : 3;
+}
 
 // How a message's scale groups tile the vector.
 struct Grouping {

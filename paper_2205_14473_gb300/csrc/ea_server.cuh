@@ -342,7 +342,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
 // compute warps decode, average, re-quantize and write e_s and the broadcast straight to HBM.
 // Used when Q_s scales are per 4096-tile (or absent) and Q_w's are per 4096-tile (or absent).
 template <int MODE, int QW, int QS>
-__global__ void __launch_bounds__(kThreads + 32, kServerMaxCtasPerSm) server_staged_kernel(const ServerArgs a)
+__global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS)) server_staged_kernel(const ServerArgs a)
 {
     extern __shared__ __align__(128) unsigned char dsm[];
     static_assert(sizeof(TileSmem) + sizeof(float) * (256 + kWorkerTab) + 128 <= kServerStaticSmem,
