@@ -132,21 +132,39 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
 // x <- x - Q_s(w) on one 4096-coordinate tile (Algorithm 1 and Algorithm 2): all loads of the
 // tile are issued first; with 4096-block scales the tile has one scale.
 // HBM traffic per coordinate: 4 B read + 4 B written + b/8 B of code.
-template <int QK, bool FULL>
-__device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile, const float *qtab)
+// x <- x - dec(Q_s message) on one tile.  BITS: the code width as a compile-time constant.  The
+// loads of x and of the raw code words are issued first; the fl(i/L) table of the uniform grid
+// (b <= 8) is built while they are in flight, and the codes are unpacked after its barrier.
+template <int QK, bool FULL, int BITS>
+__device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile, float *qtab_s)
 {
     const int64_t d = a.d;
     const Grouping &G = a.q.grp;
-    const int bits = code_bits<QK>(a.q);
+    constexpr int bits = BITS;
     const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
     const float Lf = static_cast<float>(L);
     float x[kSlots][4];
-    uint32_t c[kSlots][4];
+    uint4 raw[kSlots];  // the slot's code bits: .x for b <= 8, .x .y for b = 16, all four for b = 32
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t q = slot_of(tile, k);
         load4<FULL>(a.x, q, d, x[k]);
-        if (FULL || 4 * q < d) load_codes4(a.words, q, bits, c[k]);
+        raw[k] = make_uint4(0u, 0u, 0u, 0u);
+        if (FULL || 4 * q < d) {
+            if constexpr (bits <= 8) {
+                raw[k].x = __ldg(a.words + ((q * bits) >> 3));
+            } else if constexpr (bits == 16) {
+                const uint2 w = __ldg(reinterpret_cast<const uint2 *>(a.words) + q);
+                raw[k].x = w.x, raw[k].y = w.y;
+            } else {
+                raw[k] = __ldg(reinterpret_cast<const uint4 *>(a.words) + q);
+            }
+        }
+    }
+    const float *qtab = nullptr;
+    if constexpr (QK == QK_UNIF && bits <= 8) {
+        qtab = build_qtab<QK>(a.q, qtab_s);
+        __syncthreads();
     }
     const bool tile_scale = G.gkind == GK_BLOCK && G.G == kTile;
     const float s_tile = (has_scale<QK>() && tile_scale) ? __ldg(a.scales + tile) : 0.0f;
@@ -156,27 +174,54 @@ __device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile, con
         const int64_t q = slot_of(tile, k);
         const int64_t j0 = 4 * q;
         if (!FULL && j0 >= d) continue;
+        uint32_t c[4];
+        if constexpr (bits <= 8) {
+            const int sh = static_cast<int>((q * bits) & 7) * 4;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) c[i] = (raw[k].x >> (sh + i * bits)) & ((1u << bits) - 1u);
+        } else if constexpr (bits == 16) {
+            c[0] = raw[k].x & 0xffffu, c[1] = raw[k].x >> 16, c[2] = raw[k].y & 0xffffu, c[3] = raw[k].y >> 16;
+        } else {
+            c[0] = raw[k].x, c[1] = raw[k].y, c[2] = raw[k].z, c[3] = raw[k].w;
+        }
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             if (FULL || j0 + i < d) {
                 float s = s_tile;
                 if (has_scale<QK>() && !tile_scale) s = __ldg(a.scales + group_of(G, j0 + i, hint));
-                x[k][i] = __fsub_rn(x[k][i], decode1<QK>(c[k][i], s, a.q, Lf, L, qtab));
+                x[k][i] = __fsub_rn(x[k][i], decode1<QK>(c[i], s, a.q, Lf, L, qtab));
             }
         }
         store4<FULL>(a.x, q, d, x[k]);
     }
 }
 
+template <int QK, int BITS>
+__device__ __forceinline__ void apply_body(const ApplyArgs &a, float *qtab_s)
+{
+    const int64_t tile = blockIdx.x;
+    if ((tile + 1) * kTile <= a.d) apply_tile<QK, true, BITS>(a, tile, qtab_s);
+    else apply_tile<QK, false, BITS>(a, tile, qtab_s);
+}
+
+// One CTA per 4096-tile; the code width is dispatched once per CTA.
 template <int QK>
 __global__ void __launch_bounds__(kThreads) apply_kernel(const ApplyArgs a)
 {
     __shared__ float qtab_s[256];
-    const float *qtab = build_qtab<QK>(a.q, qtab_s);
-    if (qtab) __syncthreads();
-    const int64_t tile = blockIdx.x;
-    if ((tile + 1) * kTile <= a.d) apply_tile<QK, true>(a, tile, qtab);
-    else apply_tile<QK, false>(a, tile, qtab);
+    if constexpr (QK == QK_UNIF) {
+        switch (a.q.bits) {  // the widths ea_init accepts
+        case 2: apply_body<QK, 2>(a, qtab_s); break;
+        case 4: apply_body<QK, 4>(a, qtab_s); break;
+        case 8: apply_body<QK, 8>(a, qtab_s); break;
+        default: apply_body<QK, 16>(a, qtab_s); break;
+        }
+    } else if constexpr (QK == QK_POW2) {
+        if (a.q.bits == 4) apply_body<QK, 4>(a, qtab_s);
+        else apply_body<QK, 8>(a, qtab_s);
+    } else {
+        apply_body<QK, QK == QK_SIGN ? 1 : 32>(a, qtab_s);
+    }
 }
 
 __global__ void fill_kernel(float *p, int64_t count, float value)
