@@ -21,6 +21,9 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
             load4<FULL>(a.v, q, d, v[k]);
         }
     }
+    // the grid's fl(i/L) table, built while the loads are in flight (read after the scale
+    // reduction's barrier)
+    build_qtab<QK>(a.q, sm.qtab);
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t q = slot_of(tile, k);
@@ -57,7 +60,6 @@ __global__ void __launch_bounds__(kThreads, (MODE == MODE_S ? 4 : 3) - (QK == QK
     __shared__ TileSmem sm;
     __shared__ float4 ubuf[kSlots * kThreads];
     const int64_t tile = blockIdx.x;
-    build_qtab<QK>(a.q, sm.qtab);  // read after the scale reduction's barrier
     if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK, true>(a, tile, ubuf, sm);
     else worker_tile<MODE, QK, false>(a, tile, ubuf, sm);
 }
