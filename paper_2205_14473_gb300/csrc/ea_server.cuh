@@ -150,6 +150,18 @@ __device__ __forceinline__ bool compute_all(bool ok)
     return r != 0;
 }
 
+// Transpose the 8x8 bit matrix whose bit 8r + c is row r, column c (rows 0-3 in lo, 4-7 in hi):
+// three delta swaps of 1-, 2- and 4-bit blocks (Hacker's Delight, section 7-3).
+__device__ __forceinline__ void transpose8x8(uint32_t &lo, uint32_t &hi)
+{
+    uint32_t t;
+    t = ((lo >> 7) ^ lo) & 0x00aa00aau, lo ^= t ^ (t << 7);
+    t = ((hi >> 7) ^ hi) & 0x00aa00aau, hi ^= t ^ (t << 7);
+    t = ((lo >> 14) ^ lo) & 0x0000ccccu, lo ^= t ^ (t << 14);
+    t = ((hi >> 14) ^ hi) & 0x0000ccccu, hi ^= t ^ (t << 14);
+    t = ((hi << 4) ^ lo) & 0xf0f0f0f0u, lo ^= t, hi ^= t >> 4;
+}
+
 // Sum, in worker order, the decoded values of n workers' B-bit uniform-grid codes of this thread's
 // four slots, reading each decoded value from the per-tile table wtab (worker w's 2^B - 1 values
 // from w * 2^B); a tile's chunk holds kTile * B / 8 bytes per worker.  The worker loop is
@@ -205,13 +217,10 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
       if (a.n <= 8) {
         done = true;
         // Scaled-sign workers, n <= 8: a coordinate's average depends only on its n sign bits.
-        // Thread p forms the worker-order sum for sign pattern p, exactly as the per-coordinate
-        // loop would, divides by n, and the coordinates look their average up.  The pattern of
-        // coordinate i of a slot is gathered from X (bit 4w + i = worker w's code) by one multiply:
-        // ((X >> i) & 0x11111111) * 0x01020408 carries no bits and leaves worker w's code at bit
-        // 24 + pi(w), pi = (0, 4, 1, 5, 2, 6, 3, 7); the table is indexed in that order.
+        // Thread p forms the worker-order sum for sign pattern p (bit w = worker w's code),
+        // exactly as the per-coordinate loop would, divides by n, and the coordinates look their
+        // average up.
         {
-            // thread p's sign of worker w is bit pi(w) of p: flip[w] holds it as a binary32 sign bit
             float t = 0.0f;
 #pragma unroll
             for (int w = 0; w < 8; ++w)
@@ -221,22 +230,36 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
         // the table's barrier, and agreement on the stage wait: if any thread's wait ran out, the
         // entries just written may hold stale stage data and the tile is abandoned unread
         if (!compute_all(ok)) return false;
-        const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
+        // Patterns of eight consecutive coordinates at a time: byte b of every worker's code word
+        // (8 coordinates x 8 workers) gathered into two registers, the 8x8 bit matrix transposed,
+        // and byte j is then coordinate j's pattern.  Of a thread pair (2q, 2q+1), the even thread
+        // transposes the pair's block in slot k and the odd one in slot k+1; one shuffle swaps
+        // the halves that belong to the other thread.
         const uint32_t *c0 = reinterpret_cast<const uint32_t *>(st + P.off_codes);
+        const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
+        static_assert(kSlots % 2 == 0, "slots are taken in pairs");
+        const bool odd = threadIdx.x & 1;
+        const uint32_t bsel = (threadIdx.x >> 1) & 3;  // the block's byte in its word
+        const uint32_t sel = bsel | ((bsel + 4) << 4);
 #pragma unroll
-        for (int k = 0; k < kSlots; ++k) {
-            const int wi = (k * kThreads + static_cast<int>(threadIdx.x)) >> 3;
-            uint32_t X = 0;  // bit 4w + i = worker w's code of coordinate i of the slot
+        for (int k = 0; k < kSlots; k += 2) {
+            const int word = 32 * (k + (odd ? 1 : 0)) + static_cast<int>(threadIdx.x >> 3);
+            uint32_t wd[8];
 #pragma unroll
-            for (int w = 0; w < 8; ++w) {
-                // rotate worker w's word so that this thread's nibble lands at bits 4w .. 4w+3
-                if (w < a.n) {
-                    const uint32_t word = c0[w * (kTile / 32) + wi];
-                    X |= __funnelshift_r(word, word, (sh - 4 * w) & 31) & (0xfu << (4 * w));
-                }
+            for (int w = 0; w < 8; ++w) wd[w] = w < a.n ? c0[w * (kTile / 32) + word] : 0u;
+            uint32_t lo = __byte_perm(__byte_perm(wd[0], wd[1], sel), __byte_perm(wd[2], wd[3], sel), 0x5410);
+            uint32_t hi = __byte_perm(__byte_perm(wd[4], wd[5], sel), __byte_perm(wd[6], wd[7], sel), 0x5410);
+            transpose8x8(lo, hi);
+            const uint32_t recv = __shfl_xor_sync(0xffffffffu, odd ? lo : hi, 1);
+            const uint32_t pk = odd ? recv : lo, pk1 = odd ? hi : recv;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                // pattern byte i times 4: a byte offset into the table
+                const uint32_t o0 = (i == 0 ? pk << 2 : pk >> (8 * i - 2)) & 0x3fcu;
+                const uint32_t o1 = (i == 0 ? pk1 << 2 : pk1 >> (8 * i - 2)) & 0x3fcu;
+                acc[k][i] = *reinterpret_cast<const float *>(tb + o0);
+                acc[k + 1][i] = *reinterpret_cast<const float *>(tb + o1);
             }
-#pragma unroll
-            for (int i = 0; i < 4; ++i) acc[k][i] = wtab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
         }
       }
     }
@@ -416,13 +439,10 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
     // ------------------------------------------------------------------------- compute warps
     const int64_t d = a.d;
     // sign-pattern table (scaled-sign workers): this thread's pattern p = threadIdx.x gives worker w
-    // the sign of bit pi(w) of p, pi = (0, 4, 1, 5, 2, 6, 3, 7); kept as a binary32 sign-bit mask
+    // the sign of bit w of p, kept as a binary32 sign-bit mask
     uint32_t flip[8];
-    {
-        constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
 #pragma unroll
-        for (int w = 0; w < 8; ++w) flip[w] = ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? 0u : 0x80000000u;
-    }
+    for (int w = 0; w < 8; ++w) flip[w] = ((threadIdx.x >> w) & 1u) ? 0u : 0x80000000u;
     int64_t it = 0;
     for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
         const int s = static_cast<int>(it % S);
