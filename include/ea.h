@@ -175,6 +175,18 @@ int ea_sync_status(ea_handle *h);
 int ea_worker_compress_noalloc(const ea_config *cfg, int32_t worker, int64_t round, const float *g, float *m,
                                float *v, float *e, uint32_t *codes, float *scales, void *stream);
 
+/* Failure-detection check (no counterpart in the paper).  The staged server's waits on its
+ * shared-memory stages are bounded: after the limit the kernel records EA_E_TIMEOUT in the
+ * handle's status word, finishes its own copies and returns, and ea_sync_status reports it.  This
+ * runs that wait and that report on their own: one CTA waits on an mbarrier that nothing arrives
+ * on (arrive = 0), so the wait runs out after limit_cycles SM clock cycles, or on one that
+ * completes first (arrive = 1).  No fault, trap or unbounded loop is involved.
+ *   - limit_cycles: 1 .. 4,000,000,000 (the server's own limit, ~2 s); arrive: 0 or 1.
+ *   - stream: a cudaStream_t; the call synchronizes it.
+ *   - *timed_out: 1 if the kernel reported EA_E_TIMEOUT, else 0.
+ *   - Returns EA_E_INVAL for out-of-range arguments, EA_E_CUDA if a CUDA call fails. */
+int ea_selftest_bounded_wait(int64_t limit_cycles, int32_t arrive, void *stream, int32_t *timed_out);
+
 /* Text of the last error on h (or of the last handle-less failure when h is NULL). */
 const char *ea_last_error(const ea_handle *h);
 

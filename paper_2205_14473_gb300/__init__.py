@@ -31,7 +31,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libea.so")
 EXPORTED = ["ea_workspace_bytes", "ea_init", "ea_worker_compress", "ea_server_step", "ea_worker_apply",
             "ea_bits_sent", "ea_round_index", "ea_get_view", "ea_sync_status", "ea_last_error", "ea_destroy",
-            "ea_worker_compress_noalloc", "ea_set_hparams"]
+            "ea_worker_compress_noalloc", "ea_set_hparams", "ea_selftest_bounded_wait"]
 
 
 class EAError(RuntimeError):
@@ -82,6 +82,7 @@ def lib() -> ctypes.CDLL:
             L.ea_destroy.argtypes = [_P]
             L.ea_set_hparams.argtypes = [_P, ctypes.c_float, ctypes.c_float, ctypes.c_float]
             L.ea_worker_compress_noalloc.argtypes = [C, ctypes.c_int32, ctypes.c_int64, _P, _P, _P, _P, _P, _P, _P]
+            L.ea_selftest_bounded_wait.argtypes = [ctypes.c_int64, ctypes.c_int32, _P, ctypes.POINTER(ctypes.c_int32)]
             _lib = L
     return _lib
 
@@ -152,6 +153,13 @@ def ea_worker_compress_noalloc(cfg: ea_config, worker: int, round_index: int, g_
     """Worker compress for callers that cannot allocate (see include/ea.h): no handle, no workspace."""
     _check(lib().ea_worker_compress_noalloc(ctypes.byref(cfg), worker, round_index, g_ptr, m_ptr, v_ptr, e_ptr,
                                             codes_ptr, scales_ptr, stream_ptr))
+
+
+def ea_selftest_bounded_wait(limit_cycles: int, arrive: int, stream_ptr: int) -> bool:
+    """The server's bounded mbarrier wait on its own (see include/ea.h): True if it timed out."""
+    t = ctypes.c_int32(-1)
+    _check(lib().ea_selftest_bounded_wait(limit_cycles, arrive, stream_ptr, ctypes.byref(t)))
+    return t.value == 1
 
 
 # --------------------------------------------------------------------------- config marshalling

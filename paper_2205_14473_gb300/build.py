@@ -15,7 +15,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libea.so")
-SOURCES = ["ea_api.cu", "ea_worker.cu", "ea_noalloc.cu"] + [f"ea_server_{m}_q{q}.cu" for m in "ws" for q in range(4)]
+SOURCES = ["ea_api.cu", "ea_worker.cu", "ea_noalloc.cu", "ea_selftest.cu"] + [f"ea_server_{m}_q{q}.cu" for m in "ws" for q in range(4)]
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc")
 # binary32 per operation: no FMA contraction, IEEE division and square root, denormals kept
 FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-lineinfo", "-std=c++17", "--fmad=false",
