@@ -322,6 +322,17 @@ __device__ __forceinline__ int64_t first_group_of_tile(const Grouping &g, int64_
     return g.tile_group[tile];
 }
 
+// The group that holds every coordinate of tile `tile` (of [0, d)), or -1 when the tile spans a
+// group boundary.  Uniform over the CTA.
+__device__ __forceinline__ int64_t tile_single_group(const Grouping &g, int64_t tile, int64_t d)
+{
+    const int64_t last = min(tile * kTile + static_cast<int64_t>(kTile), d) - 1;
+    const int64_t g0 = first_group_of_tile(g, tile);
+    if (g.gkind == GK_WHOLE) return 0;
+    if (g.gkind == GK_BLOCK) return last / g.G == g0 ? g0 : -1;
+    return g.offsets[g0 + 1] > last ? g0 : -1;
+}
+
 // --------------------------------------------------------------------------------- packing
 // Coordinate j's b-bit code sits at bit j*b of the little-endian word stream.  A float4 slot q
 // (coordinates 4q .. 4q+3) spans 4b bits, so for b <= 8 it lies inside word (q*b)/8.

@@ -40,10 +40,11 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
         }
     }
 
-    // The workers' scale of a coordinate: one per worker for the whole tile when Q_w uses
-    // 4096-blocks, else a per-coordinate group lookup.
+    // The workers' scale of a coordinate: one per worker for the whole tile when the tile lies
+    // in one of Q_w's groups (always for 4096-blocks), else a per-coordinate group lookup.
     const Grouping &GW = a.qw.grp;
-    const bool wtile = GW.gkind == GK_BLOCK && GW.G == kTile;
+    const int64_t wg = has_scale<QW>() ? tile_single_group(GW, tile, d) : 0;
+    const bool wtile = wg >= 0;
     const int64_t whint = first_group_of_tile(GW, tile);
 
     float acc[kSlots][4];
@@ -56,14 +57,14 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
     for (int w = 0; w < a.n; ++w) {
         const uint32_t *ww = a.wwords + static_cast<int64_t>(w) * a.wwords_stride;
         const float *wsc = a.wscales + static_cast<int64_t>(w) * a.wscales_stride;
-        const float s_tile = (has_scale<QW>() && wtile) ? __ldg(wsc + tile) : 0.0f;
+        const float s_tile = (has_scale<QW>() && wtile) ? __ldg(wsc + wg) : 0.0f;
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
             const int64_t q = slot_of(tile, k);
             const int64_t j0 = 4 * q;
             if (j0 >= d) continue;
             uint32_t c[4];
-            load_codes4(ww, q, a.qw.bits, c);
+            load_codes4(ww, q, code_bits<QW>(a.qw), c);
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 if (j0 + i < d) {

@@ -108,6 +108,22 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
     float u[kSlots][4];
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) load4(a.buf, slot_of(tile, k), d, u[k]);
+    // a tile inside one group (the common case) has one scale: the fused tile encode
+    const int64_t g1 = tile_single_group(G, tile, d);
+    if (g1 >= 0) {
+        const float s = a.scales[g1];
+        if ((tile + 1) * kTile <= d)
+            encode_store<QK, true, true>(URegs{u}, s, tile, d, a.q, a.words, a.buf, a.ef, a.seed, a.id, a.t, qtab);
+        else
+            encode_store<QK, false, true>(URegs{u}, s, tile, d, a.q, a.words, a.buf, a.ef, a.seed, a.id, a.t, qtab);
+        if (!a.ef) {  // without error feedback the residual is 0: clear the stash of u
+            const float z[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k)
+                if (4 * slot_of(tile, k) < d) store4(a.buf, slot_of(tile, k), d, z);
+        }
+        return;
+    }
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t qs = slot_of(tile, k);
@@ -131,10 +147,8 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
     }
 }
 
-// x <- x - Q_s(w) on one 4096-coordinate tile (Algorithm 1 and Algorithm 2): all loads of the
-// tile are issued first; with 4096-block scales the tile has one scale.
-// HBM traffic per coordinate: 4 B read + 4 B written + b/8 B of code.
-// x <- x - dec(Q_s message) on one tile.  BITS: the code width as a compile-time constant.  The
+// x <- x - dec(Q_s message) on one tile (Algorithm 1 and Algorithm 2); HBM traffic per coordinate:
+// 4 B read + 4 B written + b/8 B of code.  BITS: the code width as a compile-time constant.  The
 // loads of x and of the raw code words are issued first; the fl(i/L) table of the uniform grid
 // (b <= 8) is built while they are in flight, and the codes are unpacked after its barrier.
 template <int QK, bool FULL, int BITS>
@@ -168,8 +182,9 @@ __device__ __forceinline__ void apply_tile(const ApplyArgs &a, int64_t tile, flo
         qtab = build_qtab<QK>(a.q, qtab_s);
         __syncthreads();
     }
-    const bool tile_scale = G.gkind == GK_BLOCK && G.G == kTile;
-    const float s_tile = (has_scale<QK>() && tile_scale) ? __ldg(a.scales + tile) : 0.0f;
+    const int64_t g1 = has_scale<QK>() ? tile_single_group(G, tile, d) : 0;
+    const bool tile_scale = g1 >= 0;  // one scale for the whole tile
+    const float s_tile = (has_scale<QK>() && tile_scale) ? __ldg(a.scales + g1) : 0.0f;
     const int64_t hint = first_group_of_tile(G, tile);
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
