@@ -318,7 +318,7 @@ __device__ __forceinline__ int64_t group_of(const Grouping &g, int64_t j, int64_
 __device__ __forceinline__ int64_t first_group_of_tile(const Grouping &g, int64_t tile)
 {
     if (g.gkind == GK_WHOLE) return 0;
-    if (g.gkind == GK_BLOCK) return (tile * kTile) / g.G;
+    if (g.gkind == GK_BLOCK) return g.log2G >= 0 ? (tile * kTile) >> g.log2G : (tile * kTile) / g.G;
     return g.tile_group[tile];
 }
 
@@ -326,10 +326,14 @@ __device__ __forceinline__ int64_t first_group_of_tile(const Grouping &g, int64_
 // group boundary.  Uniform over the CTA.
 __device__ __forceinline__ int64_t tile_single_group(const Grouping &g, int64_t tile, int64_t d)
 {
-    const int64_t last = min(tile * kTile + static_cast<int64_t>(kTile), d) - 1;
-    const int64_t g0 = first_group_of_tile(g, tile);
     if (g.gkind == GK_WHOLE) return 0;
-    if (g.gkind == GK_BLOCK) return last / g.G == g0 ? g0 : -1;
+    const int64_t last = min(tile * kTile + static_cast<int64_t>(kTile), d) - 1;
+    if (g.gkind == GK_BLOCK) {
+        if (g.log2G >= 12) return (tile * kTile) >> g.log2G;  // power-of-two blocks of >= 4096 hold whole tiles
+        const int64_t g0 = first_group_of_tile(g, tile);
+        return group_of(g, last, g0) == g0 ? g0 : -1;
+    }
+    const int64_t g0 = g.tile_group[tile];
     return g.offsets[g0 + 1] > last ? g0 : -1;
 }
 
