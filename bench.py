@@ -226,6 +226,23 @@ def cpu_baseline(w, placement: int, seconds: float = 12.0, blocks: int = 16):
 
 # ---------------------------------------------------------------------------------- GPU bench
 
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The job's time: the slowest rank's timed region (an all-reduce MAX when world > 1)."""
+    if world <= 1:
+        return ms
+    import torch
+
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(n: int, d: int, steps: int, world: int, t_max_ms: float) -> float:
+    """Whole-job parameter x worker elements per second: every rank runs its own replica of the
+    n-worker round on d coordinates (weak scaling), so the job processes n d steps world units."""
+    return n * d * steps * world / (t_max_ms / 1e3)
+
+
 def run_gpu(args, rank: int, world: int, local_rank: int):
     import torch
 
@@ -297,13 +314,8 @@ def run_gpu(args, rank: int, world: int, local_rank: int):
     if not args.no_e2e:
         e2e = run_e2e(args, w, rnd, x, dev, stream)
 
-    t_max = ms_total
-    if world > 1:
-        tt = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        t_max = float(tt.item())
-    units = w.n * w.d * args.steps * world
-    value = units / (t_max / 1e3)
+    t_max = max_over_ranks(ms_total, world, dev)
+    value = job_throughput(w.n, w.d, args.steps, world, t_max)
     ab = algorithmic_bytes(w, placement)
     peak, peak_kind = _peaks()
     comp_ms = statistics.mean(comp)
