@@ -53,8 +53,47 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
 
+    // Scaled-sign workers with one scale each for the tile: the worker-order sum of the first
+    // m = min(n, 8) workers depends only on their m sign bits.  Thread p forms that sum for pattern
+    // p (worker w's sign at bit pi(w), pi = (0, 4, 1, 5, 2, 6, 3, 7)) from 0, as the loop below
+    // would; a coordinate's pattern is gathered from X (bit 4w + i = worker w's code of slot
+    // coordinate i) by ((X >> i) & 0x11111111) * 0x01020408 >> 24, which carries no bits.  The
+    // remaining workers are then added in order.
+    int w_first = 0;
+    if constexpr (QW == QK_SIGN) {
+        __shared__ float stab[256];
+        if (wtile) {
+            const int m = min(a.n, 8);
+            constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
+            float t = 0.0f;
+            for (int w = 0; w < m; ++w) {
+                const float sw = __ldg(a.wscales + static_cast<int64_t>(w) * a.wscales_stride + wg);
+                t = __fadd_rn(t, ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? sw : -sw);
+            }
+            stab[threadIdx.x] = t;
+            __syncthreads();
+            const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k) {
+                const int64_t q = slot_of(tile, k);
+                if (4 * q >= d) continue;
+                uint32_t X = 0;
+#pragma unroll
+                for (int w = 0; w < 8; ++w) {
+                    if (w < m) {
+                        const uint32_t word = __ldg(a.wwords + static_cast<int64_t>(w) * a.wwords_stride + (q >> 3));
+                        X |= __funnelshift_r(word, word, (sh - 4 * w) & 31) & (0xfu << (4 * w));
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[k][i] = stab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
+            }
+            w_first = m;
+        }
+    }
+
 #pragma unroll 2
-    for (int w = 0; w < a.n; ++w) {
+    for (int w = w_first; w < a.n; ++w) {
         const uint32_t *ww = a.wwords + static_cast<int64_t>(w) * a.wwords_stride;
         const float *wsc = a.wscales + static_cast<int64_t>(w) * a.wscales_stride;
         const float s_tile = (has_scale<QW>() && wtile) ? __ldg(wsc + wg) : 0.0f;
