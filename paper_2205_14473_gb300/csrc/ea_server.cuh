@@ -254,18 +254,18 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
     // which a Q_s without scales does not have
     if constexpr (!has_scale<QS>() && (QW == QK_SIGN || QW == QK_UNIF)) compute_sync();
     if constexpr (QW == QK_SIGN) {
-      if (a.n <= 8) {
-        done = true;
-        // Scaled-sign workers, n <= 8: a coordinate's average depends only on its n sign bits.
-        // Thread p forms the worker-order sum for sign pattern p (bit w = worker w's code),
-        // exactly as the per-coordinate loop would, divides by n, and the coordinates look their
-        // average up.
+      {
+        done = a.n <= 8;
+        // Scaled-sign workers: the worker-order sum of the first m = min(n, 8) workers depends
+        // only on their m sign bits.  Thread p forms it for sign pattern p (bit w = worker w's
+        // code), exactly as the per-coordinate loop would; for n <= 8 it is divided by n and is
+        // the average, for n > 8 the remaining workers are added after it in order.
         {
             float t = 0.0f;
 #pragma unroll
             for (int w = 0; w < 8; ++w)
                 if (w < a.n) t = __fadd_rn(t, __uint_as_float(__float_as_uint(sc[w]) ^ flip[w]));
-            wtab[threadIdx.x] = pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
+            wtab[threadIdx.x] = !done ? t : pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
         }
         // the table's barrier, and agreement on the stage wait: if any thread's wait ran out, the
         // entries just written may hold stale stage data and the tile is abandoned unread
@@ -304,10 +304,14 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
       }
     }
     if (!done) {
+        // scaled-sign workers (n > 8): acc already holds the sum of workers 0..7
+        constexpr bool partial = QW == QK_SIGN;
+        if constexpr (!partial) {
 #pragma unroll
-        for (int k = 0; k < kSlots; ++k)
+            for (int k = 0; k < kSlots; ++k)
 #pragma unroll
-            for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+                for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+        }
         // Uniform-grid workers: every worker's 2L+1 decoded values s_w * fl(i/L) for this tile, as
         // decode1 would form them, so that a coordinate's decode is one table read.
         // Worker w's table starts at w * 2^b; entries 0 .. 2L = 2^b - 2 are used.
@@ -319,7 +323,8 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
                 if (i < nL) wtab[idx] = __fmul_rn(sc[idx >> bw], utab[i]);
             }
         }
-        if (!compute_all(ok)) return false;  // the table's barrier and agreement on the stage wait
+        if constexpr (!partial)
+            if (!compute_all(ok)) return false;  // the table's barrier and agreement on the stage wait
         bool summed = false;
         if constexpr (QW == QK_UNIF) {
             if (dec_tab && bw == 4) {
@@ -332,7 +337,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
         }
         if (!summed) {  // any worker count and code width; kept rolled (it is not the common case)
 #pragma unroll 1
-            for (int w = 0; w < a.n; ++w) {
+            for (int w = partial ? 8 : 0; w < a.n; ++w) {
                 const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
                 const float sw = has_scale<QW>() ? sc[w] : 0.0f;
                 const float *dw = wtab + (w << bw);
