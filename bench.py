@@ -17,6 +17,7 @@ from __future__ import annotations
 
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -84,12 +85,18 @@ def algorithmic_bytes(w, placement: int) -> dict:
             "round": n * compress + server + apply}
 
 
+_COMMENT = re.compile(r"//[^\n]*|/\*.*?\*/", re.S)
+
+
 def _kernel_source_hash() -> str:
+    """Hash of the CUDA sources with their comments removed: ncu figures taken on one version of
+    the kernels stay valid across edits that change comments only."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2205_14473_gb300", "csrc")
     for f in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, f), "rb") as fh:
-            h.update(f.encode() + fh.read())
+        with open(os.path.join(csrc, f), encoding="utf-8") as fh:
+            code = _COMMENT.sub("", fh.read())
+        h.update(f.encode() + "\n".join(ln.rstrip() for ln in code.splitlines() if ln.strip()).encode())
     return h.hexdigest()[:16]
 
 

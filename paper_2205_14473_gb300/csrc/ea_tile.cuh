@@ -1,6 +1,7 @@
 // ea_tile.cuh -- the common end of a worker or server tile: given the residual-corrected input u
-// of the tile's 4096 coordinates (held in registers, 16 per thread), form the group scale, encode
-// and pack the message, and keep the residual e = u - Q(u) (Algorithm 1 / Algorithm 2).
+// of the tile's 4096 coordinates (16 per thread, in registers or parked in shared memory), form
+// the group scale, encode and pack the message, and keep the residual e = u - Q(u) (Algorithm 1 /
+// Algorithm 2).
 #pragma once
 
 #include "ea_device.cuh"
