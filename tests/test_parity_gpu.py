@@ -73,6 +73,7 @@ _SEGS = (7, 1, 4096, 64, 5000, 3, 8192, 100, 11)
     (W.identity_q(), W.identity_q(), 1.0),                                # "Ours_full"
     (W.sign_q(4096), W.uniform_q(4, 0, True), 1.0),
     (W.identity_q(), W.sign_q(8192), 1.0),
+    (W.uniform_q(4, 6000, True), W.sign_q(6000), 1e-3),                 # blocks longer than a tile, not 2^k
 ])
 @pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
 def test_quantizer_kinds(qw, qs, gs, placement):
