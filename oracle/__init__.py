@@ -1,7 +1,7 @@
 """CPU oracle of one Efficient-Adam round (Algorithms 1 and 2 of arxiv 2205.14473).
 
-TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
-``bench.py`` may import this package.  It shares no code with the CUDA library
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline
+leg and reference arm (``--impl reference``) may import this package.  It shares no code with the CUDA library
 (``paper_2205_14473_gb300``); the two agree only through the message format and the op order that
 the header of ``ea_oracle.c`` states.
 

@@ -1,8 +1,8 @@
 /*
  * ea_oracle.c -- plain, slow CPU oracle of one Efficient-Adam round.
  *
- * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the CPU-baseline leg of
- * bench.py may load this file's library.  It shares no code, header, table or helper with the CUDA
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg
+ * and reference arm (--impl reference, the oracle timed on host cores) may load this file's library.  It shares no code, header, table or helper with the CUDA
  * library; it was written from the paper (Chen, Shen, Liu, Luo, "Efficient-Adam:
  * Communication-Efficient Distributed Adam", arxiv 2205.14473) and from the message format stated
  * below.
