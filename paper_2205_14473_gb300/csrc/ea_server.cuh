@@ -207,13 +207,54 @@ __device__ __forceinline__ void transpose8x8(uint32_t &lo, uint32_t &hi)
 // from w * 2^B); a tile's chunk holds kTile * B / 8 bytes per worker.  The worker loop is
 // kept rolled (two workers per iteration) so that the hot loop stays small in the instruction
 // cache; the slots and coordinates inside it are unrolled.
-template <int B>
+// PAIRS (B = 4): the thread-pair decode below (used with Adam at the workers; with Adam at the
+// server the per-thread form measured faster, the Adam step leaving fewer registers).
+template <int B, bool PAIRS>
 __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int n, const float *wtab,
                                                 float (&acc)[kSlots][4])
 {
     constexpr int chunk_words = kTile * B / 32;
     constexpr uint32_t mask = (1u << B) - 1u;
     // the slot's 4B bits start at bit 4 B ls of the chunk, ls = k * kThreads + threadIdx.x
+    if constexpr (B == 4 && PAIRS) {
+        // 4-bit codes, thread pairs: a code word holds the 8 coordinates of a pair (2q, 2q+1) in
+        // one slot.  The even thread decodes the pair's word in slots 0, 2, the odd one in slots 1,
+        // 3; two shift-and-masks put every code times 4 in a byte (even coordinates in a, odd in
+        // b), one byte permute per coordinate takes it out, and at the end one shuffle per
+        // coordinate hands each thread the half that is its own.
+        static_assert(kSlots % 2 == 0, "slots are taken in pairs");
+        const bool odd = threadIdx.x & 1;
+        const uint32_t *pw = reinterpret_cast<const uint32_t *>(codes) + (threadIdx.x >> 1) + (odd ? kThreads / 2 : 0);
+        const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
+        float blk[kSlots / 2][8];
+#pragma unroll
+        for (int h = 0; h < kSlots / 2; ++h)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) blk[h][j] = 0.0f;
+#pragma unroll 2
+        for (int w = 0; w < n; ++w, pw += chunk_words, tb += 4 << B) {
+#pragma unroll
+            for (int h = 0; h < kSlots / 2; ++h) {
+                const uint32_t word = pw[h * kThreads];  // slot 2h (+1 for the odd thread), word q
+                const uint32_t ev = (word << 2) & 0x3c3c3c3cu, od = (word >> 2) & 0x3c3c3c3cu;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const uint32_t o0 = __byte_perm(ev, 0u, 0x4440u | j), o1 = __byte_perm(od, 0u, 0x4440u | j);
+                    blk[h][2 * j] = __fadd_rn(blk[h][2 * j], *reinterpret_cast<const float *>(tb + o0));
+                    blk[h][2 * j + 1] = __fadd_rn(blk[h][2 * j + 1], *reinterpret_cast<const float *>(tb + o1));
+                }
+            }
+        }
+#pragma unroll
+        for (int h = 0; h < kSlots / 2; ++h)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float recv = __shfl_xor_sync(0xffffffffu, odd ? blk[h][i] : blk[h][4 + i], 1);
+                acc[2 * h][i] = odd ? recv : blk[h][i];
+                acc[2 * h + 1][i] = odd ? blk[h][4 + i] : recv;
+            }
+        return;
+    }
     const int sh = ((static_cast<int>(threadIdx.x) * B) & 7) * 4;
     const uint32_t *cw = reinterpret_cast<const uint32_t *>(codes) + ((static_cast<int>(threadIdx.x) * B) >> 3);
     const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
@@ -328,10 +369,10 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
         bool summed = false;
         if constexpr (QW == QK_UNIF) {
             if (dec_tab && bw == 4) {
-                unif_decode_sum<4>(st + P.off_codes, a.n, wtab, acc);
+                unif_decode_sum<4, MODE == MODE_W>(st + P.off_codes, a.n, wtab, acc);
                 summed = true;
             } else if (dec_tab && bw == 8) {
-                unif_decode_sum<8>(st + P.off_codes, a.n, wtab, acc);
+                unif_decode_sum<8, false>(st + P.off_codes, a.n, wtab, acc);
                 summed = true;
             }
         }
