@@ -204,12 +204,15 @@ __device__ __forceinline__ void finish_tile_smem(const float4 *ubuf, DF l1, floa
 //   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
 // BALLOT: pack 1-bit codes with __ballot_sync (worker kernels) or with shuffles (the server, whose
 // tile loop is instruction-bound).
-template <int QK, bool FULL = false, bool BALLOT = true, class USrc>
+// PASS: PASS_FUSED or PASS_STASH as a compile-time constant (the other path is then not compiled
+// in), or -1 to follow `pass`.
+template <int QK, bool FULL = false, bool BALLOT = true, int PASS = -1, class USrc>
 __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64_t d, const QParams &q,
                                             uint32_t *words, float *scales, float *resid, int ef, int pass,
                                             uint64_t seed, uint32_t id, uint32_t t, double *partials,
                                             TileSmem &sm)
 {
+    if constexpr (PASS >= 0) pass = PASS;
     if constexpr (!has_scale<QK>()) {
         encode_store<QK, FULL, BALLOT>(src, 0.0f, tile, d, q, words, resid, ef, seed, id, t, nullptr);
         return;

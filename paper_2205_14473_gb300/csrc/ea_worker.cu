@@ -6,7 +6,7 @@ namespace ea {
 // One tile of worker_kernel; FULL: the tile lies inside [0, d) (every tile but a ragged last one).
 // Each slot's u goes to ubuf (only this thread reads it again), so that no register holds u across
 // the scale's reduction and more CTAs fit on an SM.
-template <int MODE, int QK, bool FULL>
+template <int MODE, int QK, bool FULL, int PASS>
 __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, float4 *ubuf, TileSmem &sm)
 {
     const int64_t d = a.d;
@@ -41,7 +41,7 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
             store4<FULL>(a.v, q, d, v[k]);
         }
     }
-    finish_tile<QK, FULL>(USmem{ubuf}, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t,
+    finish_tile<QK, FULL, true, PASS>(USmem{ubuf}, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t,
                           a.partials, sm);
 }
 
@@ -60,8 +60,15 @@ __global__ void __launch_bounds__(kThreads, (MODE == MODE_S ? 4 : 3) - (QK == QK
     __shared__ TileSmem sm;
     __shared__ float4 ubuf[kSlots * kThreads];
     const int64_t tile = blockIdx.x;
-    if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK, true>(a, tile, ubuf, sm);
-    else worker_tile<MODE, QK, false>(a, tile, ubuf, sm);
+    // the scale pass as a compile-time constant: each instantiation carries only its own path
+    const bool full = (tile + 1) * kTile <= a.d;
+    if (a.pass == PASS_FUSED) {
+        if (full) worker_tile<MODE, QK, true, PASS_FUSED>(a, tile, ubuf, sm);
+        else worker_tile<MODE, QK, false, PASS_FUSED>(a, tile, ubuf, sm);
+    } else {
+        if (full) worker_tile<MODE, QK, true, PASS_STASH>(a, tile, ubuf, sm);
+        else worker_tile<MODE, QK, false, PASS_STASH>(a, tile, ubuf, sm);
+    }
 }
 
 // Second pass, one CTA per scale group: combine the group's per-tile partial norms in a fixed
