@@ -277,7 +277,9 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
 // One tile of the staged server on the compute warps: the stage `st` holds e_s (m_s, v_s), the
 // workers' code chunks and scales.  The stage's e_s slots then hold u until the re-quantization
 // has read it; the stage is released (arrive on `empty`) after that.
-template <int MODE, int QW, int QS, bool FULL>
+// SMALLN: n <= 8 is known at compile time (the scaled-sign table then is the whole average and the
+// per-worker path is not compiled in for scaled-sign workers).
+template <int MODE, int QW, int QS, bool FULL, bool SMALLN>
 __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
                                                    bool ok, uint64_t *empty, int Lw, float Lwf, const float *utab,
                                                    float *wtab, const uint32_t (&flip)[8], TileSmem &sm)
@@ -296,7 +298,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
     if constexpr (!has_scale<QS>() && (QW == QK_SIGN || QW == QK_UNIF)) compute_sync();
     if constexpr (QW == QK_SIGN) {
       {
-        done = a.n <= 8;
+        done = SMALLN || a.n <= 8;
         // Scaled-sign workers: the worker-order sum of the first m = min(n, 8) workers depends
         // only on their m sign bits.  Thread p forms it for sign pattern p (bit w = worker w's
         // code), exactly as the per-coordinate loop would; for n <= 8 it is divided by n and is
@@ -529,6 +531,7 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
     uint32_t flip[8];
 #pragma unroll
     for (int w = 0; w < 8; ++w) flip[w] = ((threadIdx.x >> w) & 1u) ? 0u : 0x80000000u;
+    const bool small = QW == QK_SIGN && a.n <= 8;  // full tiles of scaled-sign workers: SMALLN
     int64_t it = 0;
     for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
         const int s = static_cast<int>(it % S);
@@ -536,8 +539,9 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
         const bool ok = mbar_wait(&full[s], static_cast<uint32_t>((it / S) & 1));
         const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
         const bool go = (tile + 1) * kTile <= d
-            ? server_staged_tile<MODE, QW, QS, true>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm)
-            : server_staged_tile<MODE, QW, QS, false>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
+            ? (small ? server_staged_tile<MODE, QW, QS, true, true>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm)
+                     : server_staged_tile<MODE, QW, QS, true, false>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm))
+            : server_staged_tile<MODE, QW, QS, false, false>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
         if (!go) {
             if (threadIdx.x == 0) report_status(a.status, kStatusTimeout);
             break;
