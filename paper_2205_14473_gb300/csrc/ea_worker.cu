@@ -50,11 +50,11 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
 // with Adam at the server: u = g + e.  Then Q_w(u) and e <- u - Q_w(u) (finish_tile).
 // HBM traffic per coordinate: 16 B read + 12 B written + b/8 B of code (Adam at the worker).
 // Resident CTAs per SM the registers are sized for: four with Adam at the server (g and e per
-// coordinate), three with Adam at the worker, two for the worker-side Adam with the uniform grid
-// (stochastic rounding's draws).  Measured: the server-side-Adam uniform grid runs faster at four
-// CTAs with a few bytes of spill than at three without.
+// coordinate), three with Adam at the worker.  Measured: the server-side-Adam uniform grid runs
+// faster at four CTAs with a few bytes of spill than at three without, and the worker-side-Adam
+// uniform grid faster at three (80 registers, a few bytes of spill) than at two.
 template <int MODE, int QK>
-__global__ void __launch_bounds__(kThreads, (MODE == MODE_S ? 4 : 3) - (QK == QK_UNIF && MODE == MODE_W ? 1 : 0))
+__global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 3)
     worker_kernel(const WorkerArgs a)
 {
     __shared__ TileSmem sm;
