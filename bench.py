@@ -173,9 +173,10 @@ class OracleSample:
     """The oracle, as it stands, on a bounded sample of the workload: `blocks` whole 4096-blocks of
     every worker when the scales are per 4096-block (the round is separable by block; the global
     coordinates key the Philox counters), else a prefix of d with the same quantizers.  One step()
-    is one full round (n worker steps, the server step, the update of x) on one host thread."""
+    is one full round (n worker steps, the server step, the update of x) on `threads` host threads
+    (the workers, and chunks of whole scale groups, run concurrently)."""
 
-    def __init__(self, w, placement: int, blocks: int = 16):
+    def __init__(self, w, placement: int, blocks: int = 16, threads: int = 1):
         import numpy as np
 
         import oracle as O
@@ -202,7 +203,8 @@ class OracleSample:
 
         self.d, self.n = d, w.n
         self.orc = O.OracleRound(d, w.n, quant(w.qw), quant(w.qs), w.alpha, w.beta1, w.beta2, w.eps,
-                                 seed=w.seed, mode=placement, gidx=gidx, threads=1)
+                                 seed=w.seed, mode=placement, gidx=gidx, threads=threads)
+        self.threads = threads
         rng = np.random.default_rng(0)
         self.grads = [(rng.standard_normal(d) * w.grad_std).astype(np.float32) for _ in range(w.n)]
         self.x = np.zeros(d, np.float32)
@@ -217,9 +219,16 @@ class OracleSample:
         return self.n * self.d
 
 
-def cpu_baseline(w, placement: int, seconds: float = 12.0, blocks: int = 16):
-    """Oracle rounds on the sample, repeated for about `seconds` of CPU work."""
-    ob = OracleSample(w, placement, blocks)
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def _oracle_rate(w, placement: int, seconds: float, blocks: int, threads: int):
+    ob = OracleSample(w, placement, blocks, threads)
+    ob.step()  # warm-up (page-in of the sample's arrays)
     rounds, t0 = 0, time.perf_counter()
     while True:
         ob.step()
@@ -227,8 +236,20 @@ def cpu_baseline(w, placement: int, seconds: float = 12.0, blocks: int = 16):
         el = time.perf_counter() - t0
         if el >= seconds:
             break
-    return {"value": rounds * ob.units_per_step / el, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{ob.sample}; {rounds} rounds in {el:.1f} s, single-threaded C oracle"}
+    return rounds * ob.units_per_step / el, f"{ob.sample}; {rounds} rounds in {el:.1f} s"
+
+
+def cpu_baseline(w, placement: int, seconds: float = 12.0):
+    """The oracle, as it stands, on a bounded sample of the workload, timed on this host's cores:
+    one thread per worker (n threads: the workers concurrently, then the server step and the update
+    of x over chunks of whole scale groups), and on one core for comparison."""
+    cores = host_cores()
+    threads = max(1, min(w.n, cores))
+    val, sample = _oracle_rate(w, placement, seconds / 2, 1024, threads)
+    val1, sample1 = _oracle_rate(w, placement, seconds / 2, 128, 1)
+    return {"value": val, "unit": UNIT, "cores": threads, "threads": threads, "cores_available": cores,
+            "kind": "oracle", "sample": f"{sample}, {threads} host threads (one per worker)",
+            "value_1core": val1, "sample_1core": f"{sample1}, one host thread"}
 
 
 # ---------------------------------------------------------------------------------- GPU bench
@@ -250,90 +271,148 @@ def job_throughput(n: int, d: int, steps: int, world: int, t_max_ms: float) -> f
     return n * d * steps * world / (t_max_ms / 1e3)
 
 
+NOMINAL_HBM_GBS = 8000.0  # the GB300's nominal ~8 TB/s, the reference of the 70% target
+
+
+def _launches_per_round(w) -> int:
+    """Library kernel launches per round: one per message, plus finalize + encode when the message's
+    scale groups span tiles (the two-pass scale), plus the apply."""
+    from paper_2205_14473_gb300 import workloads as W
+
+    def per_message(spec):
+        has_scale = spec.kind in (W.Q_SIGN_L1, W.Q_UNIFORM_MAX)
+        one_pass = spec.group == 4096 or ((spec.group == 0 or spec.group >= w.d) and w.d <= 4096)
+        return 1 if (not has_scale or one_pass) else 3
+    return w.n * per_message(w.qw) + per_message(w.qs) + 1
+
+
+class RoundTimer:
+    """A workload's round state on one device (library handle with its workspace, n resident
+    gradients, x) and CUDA-event timing of its rounds on the library's stream."""
+
+    def __init__(self, w, placement: int, dev, stream):
+        import torch
+
+        import paper_2205_14473_gb300 as ea
+        from paper_2205_14473_gb300 import workloads as W
+
+        self.w, self.placement, self.dev, self.stream = w, placement, dev, stream
+        cfg = ea.EAConfig.from_workload(w, placement=placement)
+        with torch.cuda.stream(stream):
+            self.rnd = ea.EARound(cfg, stream=stream, device=dev)
+            self.grads = [torch.empty(w.d, dtype=torch.float32, device=dev) for _ in range(w.n)]
+            for i, g in enumerate(self.grads):
+                W.gradient_device(w, i, 0, g)
+            self.x = torch.zeros(w.d, dtype=torch.float32, device=dev)
+        stream.synchronize()
+
+    def one_round(self, ev=None):
+        w, rnd, s = self.w, self.rnd, self.stream
+        for i in range(w.n):
+            if ev is not None:
+                ev["c0"][i].record(s)
+            rnd.worker_compress(i, self.grads[i])
+            if ev is not None:
+                ev["c1"][i].record(s)
+        if ev is not None:
+            ev["s0"].record(s)
+        rnd.server_step()
+        if ev is not None:
+            ev["s1"].record(s)
+        rnd.apply(self.x)
+        if ev is not None:
+            ev["a1"].record(s)
+
+    def run(self, steps: int, warmup: int, barrier=lambda: None, clocks=None):
+        """warmup untimed rounds, then `steps` rounds between two events (per-kernel events inside);
+        returns (total ms, per-launch ms lists)."""
+        import torch
+
+        for _ in range(warmup):
+            self.one_round()
+        self.stream.synchronize()
+        E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+        per = [{"c0": [E() for _ in range(self.w.n)], "c1": [E() for _ in range(self.w.n)], "s0": E(), "s1": E(),
+                "a1": E()} for _ in range(steps)]
+        start, end = E(), E()
+        if clocks is not None:
+            time.sleep(0.3)
+        barrier()
+        torch.cuda.synchronize(self.dev)
+        start.record(self.stream)
+        for k in range(steps):
+            self.one_round(per[k])
+        end.record(self.stream)
+        torch.cuda.synchronize(self.dev)
+        barrier()
+        comp = [ev["c0"][i].elapsed_time(ev["c1"][i]) for ev in per for i in range(self.w.n)]
+        serv = [ev["s0"].elapsed_time(ev["s1"]) for ev in per]
+        appl = [ev["s1"].elapsed_time(ev["a1"]) for ev in per]
+        self.rnd.sync()
+        return start.elapsed_time(end), comp, serv, appl
+
+    def kernel_figures(self, ms_total: float, steps: int, comp, serv, appl) -> dict:
+        """Per-kernel mean times and algorithmic GB/s, against the measured copy peak and 8 TB/s."""
+        ab = algorithmic_bytes(self.w, self.placement)
+        peak, _ = _peaks()
+        out = {"workload": self.w.name, "placement": "worker" if self.placement == 0 else "server",
+               "d": self.w.d, "n_workers": self.w.n, "steps": steps, "ms_per_round": ms_total / steps,
+               "elems_per_s": self.w.n * self.w.d * steps / (ms_total / 1e3)}
+        for name, ts in (("compress", comp), ("server", serv), ("apply", appl)):
+            ms = statistics.mean(ts)
+            gbs = ab[name] / (ms / 1e3) / 1e9
+            out[name] = {"ms": ms, "min_ms": min(ts), "gbs": gbs, "frac_measured": gbs / peak,
+                         "frac_8tbs": gbs / NOMINAL_HBM_GBS, "bytes": ab[name]}
+        rgbs = ab["round"] / (ms_total / steps / 1e3) / 1e9
+        out["round"] = {"gbs": rgbs, "frac_measured": rgbs / peak, "frac_8tbs": rgbs / NOMINAL_HBM_GBS,
+                        "bytes": ab["round"]}
+        return out
+
+    def free(self):
+        import torch
+
+        self.rnd = self.grads = self.x = None
+        torch.cuda.synchronize(self.dev)
+        torch.cuda.empty_cache()
+
+
+# The other workloads and placements timed after the headline line (each alone on the device, its
+# workspace freed before the next): the placement trade-off and the per-kernel rates at c3 and c4.
+EXTRA_CONFIGS = [("c5", 1), ("c4", 0), ("c4", 1), ("c3", 0), ("c3", 1)]
+
+
 def run_gpu(args, rank: int, world: int, local_rank: int):
     import torch
 
-    import paper_2205_14473_gb300 as ea
     from paper_2205_14473_gb300 import build as B
-    from paper_2205_14473_gb300 import workloads as W
 
     B.build()
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     w = _workload(args.workload)
     placement = 0 if args.placement == "worker" else 1
-    cfg = ea.EAConfig.from_workload(w, placement=placement)
     stream = torch.cuda.Stream(dev)
-    with torch.cuda.stream(stream):
-        rnd = ea.EARound(cfg, stream=stream, device=dev)
-        grads = [torch.empty(w.d, dtype=torch.float32, device=dev) for _ in range(w.n)]
-        for i, g in enumerate(grads):
-            W.gradient_device(w, i, 0, g)
-        x = torch.zeros(w.d, dtype=torch.float32, device=dev)
-    stream.synchronize()
-
-    def one_round(events=None):
-        for i in range(w.n):
-            if events is not None:
-                events["c0"][i].record(stream)
-            rnd.worker_compress(i, grads[i])
-            if events is not None:
-                events["c1"][i].record(stream)
-        if events is not None:
-            events["s0"].record(stream)
-        rnd.server_step()
-        if events is not None:
-            events["s1"].record(stream)
-        rnd.apply(x)
-        if events is not None:
-            events["a1"].record(stream)
-
-    for _ in range(args.warmup):
-        one_round()
-    stream.synchronize()
-
-    def mk():
-        E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-        return {"c0": [E() for _ in range(w.n)], "c1": [E() for _ in range(w.n)], "s0": E(), "s1": E(), "a1": E()}
-
-    per_step = [mk() for _ in range(args.steps)]
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    rt = RoundTimer(w, placement, dev, stream)
     barrier = (lambda: torch.distributed.barrier()) if world > 1 else (lambda: None)
     with ClockSampler(local_rank) as clk:
-        time.sleep(0.3)
-        barrier()
-        torch.cuda.synchronize(dev)
-        start.record(stream)
-        for k in range(args.steps):
-            one_round(per_step[k])
-        end.record(stream)
-        torch.cuda.synchronize(dev)
-        barrier()
-    ms_total = start.elapsed_time(end)
-    comp = [ev["c0"][i].elapsed_time(ev["c1"][i]) for ev in per_step for i in range(w.n)]
-    serv = [ev["s0"].elapsed_time(ev["s1"]) for ev in per_step]
-    appl = [ev["s1"].elapsed_time(ev["a1"]) for ev in per_step]
-    rnd.sync()
+        ms_total, comp, serv, appl = rt.run(args.steps, args.warmup, barrier, clocks=clk)
+    figs = rt.kernel_figures(ms_total, args.steps, comp, serv, appl)
 
-    # ---- end to end through the C-ABI with host buffers: H2D of every worker's gradient from pinned
-    # host memory, the round, D2H of x; copies overlap the previous worker's compress on a copy stream
+    # ---- end to end through the C-ABI with host buffers (pinned gradients read over the host link,
+    # the broadcast message read back every step)
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, w, rnd, x, dev, stream)
+        e2e = run_e2e(args, w, rt.rnd, rt.x, dev, stream)
+    rnd_ws = rt.rnd.workspace_bytes
+    rt.free()
 
     t_max = max_over_ranks(ms_total, world, dev)
     value = job_throughput(w.n, w.d, args.steps, world, t_max)
     ab = algorithmic_bytes(w, placement)
     peak, peak_kind = _peaks()
-    comp_ms = statistics.mean(comp)
+    comp_ms = figs["compress"]["ms"]
     achieved = ab["compress"] / (comp_ms / 1e3) / 1e9
     traffic = _ncu_traffic("worker_kernel", w.name, placement)
-    def launches(spec):  # one kernel, plus finalize + encode when the scale groups span tiles
-        has_scale = spec.kind in (W.Q_SIGN_L1, W.Q_UNIFORM_MAX)
-        one_pass = spec.group == 4096 or ((spec.group == 0 or spec.group >= w.d) and w.d <= 4096)
-        return 1 if (not has_scale or one_pass) else 3
-    launches_per_round = w.n * launches(w.qw) + launches(w.qs) + 1
-    rnd_ws = rnd.workspace_bytes
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True,
@@ -344,16 +423,35 @@ def run_gpu(args, rank: int, world: int, local_rank: int):
                    "placement": "worker" if placement == 0 else "server"},
         "roofline": {"bound": "hbm", "kernel": "worker_kernel (compress)", "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak, "traffic": traffic,
-                     "algorithmic_bytes_per_launch": ab["compress"]},
-        "kernels_ms": {"compress_mean": comp_ms, "compress_min": min(comp), "server_mean": statistics.mean(serv),
-                       "apply_mean": statistics.mean(appl),
-                       "server_gbs": ab["server"] / (statistics.mean(serv) / 1e3) / 1e9,
-                       "apply_gbs": ab["apply"] / (statistics.mean(appl) / 1e3) / 1e9,
-                       "round_gbs": ab["round"] / (t_max / args.steps / 1e3) / 1e9},
-        "gpu_launches": launches_per_round * args.steps,
+                     "algorithmic_bytes_per_launch": ab["compress"],
+                     "peak_nominal": NOMINAL_HBM_GBS, "frac_nominal": achieved / NOMINAL_HBM_GBS,
+                     "note": "peak = the driver-measured copy bandwidth (a torch copy), which a streaming "
+                             "kernel can exceed; frac_nominal is against the GB300's nominal ~8 TB/s"},
+        "kernels_ms": {"compress_mean": comp_ms, "compress_min": figs["compress"]["min_ms"],
+                       "server_mean": figs["server"]["ms"], "apply_mean": figs["apply"]["ms"],
+                       "server_gbs": figs["server"]["gbs"], "apply_gbs": figs["apply"]["gbs"],
+                       "round_gbs": figs["round"]["gbs"],
+                       "server_frac_8tbs": figs["server"]["frac_8tbs"],
+                       "compress_frac_8tbs": figs["compress"]["frac_8tbs"]},
+        "gpu_launches": _launches_per_round(w) * args.steps,
         "clocks": clk.summary(),
         "e2e": e2e,
     }
+    if not args.no_extra and world == 1 and not _OVERRIDE:
+        extra = {}
+        for name, pl in EXTRA_CONFIGS:
+            if (name, pl) == (w.name, placement):
+                continue
+            we = _workload(name)
+            rte = RoundTimer(we, pl, dev, stream)
+            with ClockSampler(local_rank) as clk2:
+                ms, c, sv, ap = rte.run(args.extra_steps, max(3, args.warmup), clocks=clk2)
+            f = rte.kernel_figures(ms, args.extra_steps, c, sv, ap)
+            f["clocks"] = clk2.summary()
+            f["gpu_launches"] = _launches_per_round(we) * args.extra_steps
+            extra[f"{name}/{'W' if pl == 0 else 'S'}"] = f
+            rte.free()
+        out["configs"] = extra
     return out
 
 
@@ -458,6 +556,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--d", type=int, default=None, help="override d (small profiling cases)")
     ap.add_argument("--n", type=int, default=None, help="override the worker count")
+    ap.add_argument("--no-extra", action="store_true", help="time the headline workload only")
+    ap.add_argument("--extra-steps", type=int, default=10, help="timed rounds of each extra workload")
     args = ap.parse_args()
 
     if args.d:
@@ -477,7 +577,9 @@ def main():
         import oracle
 
         oracle.build()
-        ob = OracleSample(w, placement, blocks=64)
+        cores = host_cores()
+        threads = max(1, min(w.n, cores))
+        ob = OracleSample(w, placement, blocks=1024, threads=threads)
         for _ in range(args.warmup):
             ob.step()
         t0 = time.perf_counter()
@@ -485,8 +587,9 @@ def main():
             ob.step()
         el = time.perf_counter() - t0
         val = args.steps * ob.units_per_step / el
-        cb = {"value": val, "unit": UNIT, "cores": 1, "kind": "oracle",
-              "sample": f"{ob.sample}; {args.steps} timed rounds in {el:.2f} s, single-threaded C oracle"}
+        cb = {"value": val, "unit": UNIT, "cores": threads, "threads": threads, "cores_available": cores,
+              "kind": "oracle",
+              "sample": f"{ob.sample}; {args.steps} timed rounds in {el:.2f} s, {threads} host threads (one per worker)"}
         out = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": 1,
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",

@@ -167,8 +167,9 @@ int ea_sync_status(ea_handle *h);
  *     v = eps (0 with adam_form 1), e = 0 as Algorithm 2 does.  codes: device, 16-byte aligned, room for
  *     4 * ceil(d * bits / 128) words; scales: device, one binary32.  round: the 0-based round,
  *     which with `worker` and cfg->seed keys the stochastic rounding.  stream: a cudaStream_t.
- *   - The first call on each device looks up the scratch array's device address (with that
- *     device current); make that first call before any stream capture.
+ *   - Every call looks up the scratch array's device address in the current device's context
+ *     (cudaGetSymbolAddress, which allocates nothing); the first call on a device may also load
+ *     the library's module there, so make that first call before any stream capture.
  *   - Every call shares the one array, which keeps the last call's contents; the calls rewrite all
  *     of it that they read.  Calls that overlap on the GPU race: order them on one stream or with
  *     events. */

@@ -199,6 +199,91 @@ class OracleRound:
         self.threads = max(1, int(threads))
         self._scratch = [(np.zeros(d, f32), np.zeros(d, f32)) for _ in range(n)]
         self._sscratch = (np.zeros(d, f32), np.zeros(d, f32), np.zeros(d, f32))
+        self._chunks = self._make_chunks() if self.threads > 1 else []
+        self._pool = _futures.ThreadPoolExecutor(self.threads) if self.threads > 1 else None
+
+    # ------------------------------------------------------------------------ chunked execution
+    # The round is separable by scale group: every coordinate's arithmetic depends only on its own
+    # values and on its groups' scales.  With threads > 1, the vector is cut into chunks at offsets
+    # that are group boundaries of both quantizers and start whole code words of both messages, and
+    # the C steps run on the chunks concurrently (the same functions, on sub-arrays; global indices
+    # key the Philox counters).  Whole-vector groups cannot be cut: they run as one chunk.
+
+    def _make_chunks(self):
+        d, qw, qs = self.d, self.qw, self.qs
+        cand = None
+        for q in (qw, qs):
+            if q.has_scales:
+                offs = set(int(o) for o in q.offsets[1:-1])
+                cand = offs if cand is None else cand & offs
+        if cand is None:
+            cand = set(range(1024, d, 1024))
+        cand = sorted(o for o in cand if (o * qw.bits) % 32 == 0 and (o * qs.bits) % 32 == 0)
+        k = min(4 * self.threads, 64)
+        cuts = [0]
+        for j in range(1, k):
+            target = d * j // k
+            i = int(np.searchsorted(cand, target))
+            near = [cand[i2] for i2 in (i - 1, i) if 0 <= i2 < len(cand)]
+            best = min(near, key=lambda c: abs(c - target), default=None)
+            if best is not None and best > cuts[-1]:
+                cuts.append(best)
+        cuts.append(d)
+        if len(cuts) <= 2:
+            return []
+        gidx = self.gidx if self.gidx is not None else (
+            np.arange(d, dtype=np.int64) if (qw.stochastic or qs.stochastic) else None)
+        chunks = []
+        for lo, hi in zip(cuts[:-1], cuts[1:]):
+            def sub(q):
+                if not q.has_scales:
+                    return Quantizer(q.kind, q.bits, np.array([0, hi - lo], np.int64), q.stochastic, q.pow2_k,
+                                     q.pow2_K), 0
+                g0 = int(np.searchsorted(q.offsets, lo))
+                g1 = int(np.searchsorted(q.offsets, hi))
+                return Quantizer(q.kind, q.bits, q.offsets[g0:g1 + 1] - lo, q.stochastic, q.pow2_k, q.pow2_K), g0
+            (qwc, gw), (qsc, gs) = sub(qw), sub(qs)
+            gi = None if gidx is None else np.ascontiguousarray(gidx[lo:hi])
+            chunks.append((lo, hi, qwc, gw, qsc, gs, gi))
+        return chunks
+
+    def _cfg_for(self, d: int):
+        c = self.cfg
+        return _Config(d, c.n, c.mode, c.error_feedback, c.adam_form, c.alpha, c.beta1, c.beta2, c.eps, c.seed)
+
+    @staticmethod
+    def _at(a: np.ndarray, off: int):
+        """Pointer to element `off` of a C-contiguous 1-D array."""
+        return ctypes.c_void_p(a.ctypes.data + off * a.itemsize)
+
+    def _worker_chunk(self, i: int, g: np.ndarray, ch) -> None:
+        lo, hi, qwc, gw, _, _, gi = ch
+        u, dec = self._scratch[i]
+        W = self.mode == ADAM_AT_WORKER
+        cfg = self._cfg_for(hi - lo)
+        lib().ora_worker_step(ctypes.byref(cfg), ctypes.byref(qwc._c), _ptr(gi), i, self.t, self._at(g, lo),
+                              self._at(self.m[i], lo) if W else None, self._at(self.v[i], lo) if W else None,
+                              self._at(self.e[i], lo), self._at(u, lo), self._at(dec, lo),
+                              self._at(self.wwords[i], lo * self.qw.bits // 32), self._at(self.wscales[i], gw))
+
+    def _server_chunk(self, ch) -> None:
+        lo, hi, qwc, gw, qsc, gs, gi = ch
+        bw = self.qw.bits
+        ww = (ctypes.c_void_p * self.n)(*[self.wwords[i].ctypes.data + (lo * bw // 32) * 4 for i in range(self.n)])
+        ws = (ctypes.c_void_p * self.n)(*[self.wscales[i].ctypes.data + gw * 4 for i in range(self.n)])
+        acc, w, dec = self._sscratch
+        S = self.mode == ADAM_AT_SERVER
+        cfg = self._cfg_for(hi - lo)
+        lib().ora_server_step(ctypes.byref(cfg), ctypes.byref(qwc._c), ctypes.byref(qsc._c), _ptr(gi), self.t,
+                              ctypes.cast(ww, _P), ctypes.cast(ws, _P), self._at(self.es, lo),
+                              self._at(self.ms, lo) if S else None, self._at(self.vs, lo) if S else None,
+                              self._at(acc, lo), self._at(w, lo), self._at(dec, lo),
+                              self._at(self.swords, lo * self.qs.bits // 32), self._at(self.sscales, gs))
+
+    def _apply_chunk(self, x: np.ndarray, ch) -> None:
+        lo, hi, _, _, qsc, gs, _ = ch
+        lib().ora_apply(ctypes.byref(qsc._c), hi - lo, self._at(self.swords, lo * self.qs.bits // 32),
+                        self._at(self.sscales, gs), self._at(x, lo), self._at(self._sscratch[2], lo))
 
     def set_hparams(self, alpha: float, beta1: float, beta2: float) -> None:
         """alpha_t, beta and theta_t for the following rounds (schedules such as Assumption 2's)."""
@@ -215,15 +300,27 @@ class OracleRound:
                               _ptr(self.wwords[i]), _ptr(self.wscales[i]))
 
     def compress_all(self, gs) -> None:
-        """All n workers; with threads > 1 the workers run concurrently (one host thread each)."""
+        """All n workers; with threads > 1 the workers (and chunks of whole scale groups of each
+        worker's vector, where the groups allow it) run concurrently on host threads."""
         if self.threads == 1:
             for i in range(self.n):
                 self.worker_compress(i, gs[i])
             return
-        with _futures.ThreadPoolExecutor(self.threads) as ex:
-            list(ex.map(lambda i: self.worker_compress(i, gs[i]), range(self.n)))
+        if not self._chunks:
+            list(self._pool.map(lambda i: self.worker_compress(i, gs[i]), range(self.n)))
+            return
+        gs = [np.ascontiguousarray(g, dtype=np.float32) for g in gs]
+        assert all(g.shape == (self.d,) for g in gs)
+        tasks = [(i, ch) for i in range(self.n) for ch in self._chunks]
+        list(self._pool.map(lambda a: self._worker_chunk(a[0], gs[a[0]], a[1]), tasks))
 
     def server_step(self) -> None:
+        if self._chunks:
+            list(self._pool.map(self._server_chunk, self._chunks))
+            self.up_bits += self.n * self.qw.message_bits(self.d)
+            self.down_bits += self.n * self.qs.message_bits(self.d)
+            self.t += 1
+            return
         ww = (ctypes.c_void_p * self.n)(*[self.wwords[i].ctypes.data for i in range(self.n)])
         ws = (ctypes.c_void_p * self.n)(*[self.wscales[i].ctypes.data for i in range(self.n)])
         acc, w, dec = self._sscratch
@@ -239,6 +336,9 @@ class OracleRound:
 
     def apply(self, x: np.ndarray) -> None:
         assert x.dtype == np.float32 and x.flags["C_CONTIGUOUS"] and x.shape == (self.d,)
+        if self._chunks:
+            list(self._pool.map(lambda ch: self._apply_chunk(x, ch), self._chunks))
+            return
         dec = self._sscratch[2]
         lib().ora_apply(ctypes.byref(self.qs._c), self.d, _ptr(self.swords), _ptr(self.sscales),
                         _ptr(x), _ptr(dec))

@@ -21,6 +21,8 @@ constexpr uint32_t kServerMaxDynSmem = 200 * 1024;
 constexpr uint32_t kSmemPerSm = 228 * 1024;
 constexpr uint32_t kSmemReservedPerCta = 1024;
 constexpr int kWarps = kThreads / 32;
+// Device ordinals for which per-device host state (kernel attributes) is kept.
+constexpr int kMaxDevices = 64;
 
 enum QKind : int { QK_IDENT = 0, QK_SIGN = 1, QK_UNIF = 2, QK_POW2 = 3 };
 enum GKind : int { GK_WHOLE = 0, GK_BLOCK = 1, GK_SEG = 2 };

@@ -14,7 +14,6 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
-#include <mutex>
 
 #include "ea.h"
 #include "ea_internal.h"
@@ -24,13 +23,8 @@ namespace {
 using namespace ea;
 
 constexpr int64_t kMaxTiles = EA_NOALLOC_MAX_D / kTile;
-constexpr int kMaxDevices = 64;
-
 // [0, 16): the two offsets of the single scale group's partial norms; [256, ...): the partials.
 __device__ __align__(256) unsigned char g_scratch[256 + kMaxTiles * sizeof(double)];
-
-std::mutex g_mu;
-unsigned char *g_scratch_addr[kMaxDevices] = {};
 
 __global__ void write_group_offsets(int64_t *pair_base, int64_t n_tiles)
 {
@@ -51,21 +45,15 @@ int fail(int code, const char *fmt, ...)
     return code;
 }
 
-// The device address of g_scratch on the current device, looked up once per device.
+// The device address of g_scratch in the current context, looked up on every call: the lookup
+// allocates nothing, and a cached address would go stale after cudaDeviceReset or when another
+// context is made current on the same device.
 int scratch_address(unsigned char **out)
 {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return fail(EA_E_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
-    if (dev < 0 || dev >= kMaxDevices) return fail(EA_E_UNSUPPORTED, "device %d beyond %d", dev, kMaxDevices);
-    std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_scratch_addr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_scratch);
-        if (e != cudaSuccess) return fail(EA_E_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
-        g_scratch_addr[dev] = static_cast<unsigned char *>(p);
-    }
-    *out = g_scratch_addr[dev];
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
+    if (e != cudaSuccess) return fail(EA_E_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+    *out = static_cast<unsigned char *>(p);
     return EA_OK;
 }
 

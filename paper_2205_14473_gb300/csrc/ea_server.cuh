@@ -1,6 +1,8 @@
 // ea_server.cuh -- the server's round (Algorithm 1) on one 4096-coordinate tile.
 #pragma once
 
+#include <atomic>
+
 #include "ea_async.cuh"
 #include "ea_tile.cuh"
 
@@ -552,15 +554,21 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
 template <int MODE, int QW, int QS>
 static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
 {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kServerMaxDynSmem);
+    // Function attributes are per device: one flag per device ordinal.  Two threads that race on a
+    // first launch both set the same values, which is harmless.
+    static std::atomic<bool> attr_set[kMaxDevices];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    if (!attr_set[dev].load(std::memory_order_acquire)) {
+        e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kServerMaxDynSmem);
         if (e == cudaSuccess)  // all of the SM's unified L1 / shared memory as shared memory
             e = cudaFuncSetAttribute(server_staged_kernel<MODE, QW, QS>,
                                      cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_set[dev].store(true, std::memory_order_release);
     }
     server_staged_kernel<MODE, QW, QS><<<a.plan.grid, kThreads + 32, a.plan.smem_bytes, s>>>(a);
     return cudaGetLastError();

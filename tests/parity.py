@@ -2,21 +2,30 @@
 rounds on the same seeded inputs, each from its own state; after every round every output is
 compared.  Nothing computed by the CUDA path is ever fed to the oracle.
 
-Tolerances (the contract of this port):
-  * codes: bit-exact, except at coordinates whose quantizer input lies within 2 ulp (of the
-    larger of the two terms that formed it) of a decision threshold; at most 1e-6 of all
-    coordinates (rounded down, at least the ones so flagged) may differ, and a coordinate that
-    differed is excluded, with its scale groups, from later comparisons;
+Tolerances:
+  * codes: the contract allows a code to differ only where the quantizer's input lies within 2 ulp
+    of a decision threshold (the input margin 2 ulp(max(|step|, |e_old|)), carried to the decision
+    variable: for Example 1's grid that is y = u L / s, so the window is margin * L / s, and nothing
+    more), at no more than 1e-6 of the positions.  The tests hold the stronger claim that no code
+    differs at all: with `strict` (the default) any code mismatch fails the test, and its message
+    says whether the position was inside that window.  Without `strict`, a mismatch inside the
+    window is counted and its coordinate is excluded from later comparisons; a later scale that
+    differs is then accepted only for a group that holds such a coordinate (and that group is then
+    excluded too);
   * scales: within 1e-6 relative;
   * x, m, v and residuals: |gpu - oracle| <= 1e-7 + 1e-5 |oracle| elementwise;
   * bits sent: exactly equal.
 
+Every Lockstep records what it compared (rounds, code positions, state values, mismatches) in
+RUNS; tests/conftest.py prints the totals at the end of the session.
+
 Large workloads whose scale groups are blocks or tensors are separable by group: there the oracle
-runs on a fixed sample of whole groups (global coordinates kept for the Philox counters).
+may run on a fixed sample of whole groups (global coordinates kept for the Philox counters).
 """
 from __future__ import annotations
 
 import dataclasses
+import os
 
 import numpy as np
 import torch
@@ -26,6 +35,16 @@ import paper_2205_14473_gb300 as ea
 from paper_2205_14473_gb300 import workloads as W
 
 ATOL, RTOL, SCALE_RTOL = 1e-7, 1e-5, 1e-6
+
+RUNS: list[dict] = []  # one record per Lockstep, for the session summary
+
+
+def host_threads() -> int:
+    """Host cores this process may use (the oracle's thread count)."""
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except AttributeError:
+        return max(1, os.cpu_count() or 1)
 
 
 def _agree(g: torch.Tensor, w: torch.Tensor, rtol: float, atol: float) -> torch.Tensor:
@@ -63,8 +82,10 @@ class RoundReport:
 
 
 class Lockstep:
-    def __init__(self, cfg: ea.EAConfig, sample_groups=None, threads: int = 8):
+    def __init__(self, cfg: ea.EAConfig, sample_groups=None, threads: int | None = None, strict: bool = True):
+        threads = host_threads() if threads is None else threads
         self.cfg = cfg
+        self.strict = strict
         self.dev = torch.device("cuda", torch.cuda.current_device())
         self.gpu = ea.EARound(cfg)
         d = cfg.d
@@ -99,6 +120,10 @@ class Lockstep:
         self.tainted = torch.zeros(self.d_o, dtype=torch.bool, device=self.dev)
         self.total_mismatch = 0
         self.reports: list[RoundReport] = []
+        self.record = {"test": os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0], "d": cfg.d, "n": cfg.n,
+                       "d_oracle": self.d_o, "rounds": 0, "code_positions": 0, "values": 0, "scales": 0,
+                       "mismatches": 0, "flagged": 0}
+        RUNS.append(self.record)
 
     def set_hparams(self, alpha: float, beta1: float, beta2: float) -> None:
         self.gpu.set_hparams(alpha, beta1, beta2)
@@ -127,6 +152,7 @@ class Lockstep:
         rep = RoundReport(self.orc.t)
         self._compare(rep, e_old, es_old, x_dev, x_host)
         self.reports.append(rep)
+        self.record["rounds"] += 1
         return rep
 
     # ------------------------------------------------------------------------------- comparisons
@@ -141,6 +167,7 @@ class Lockstep:
         g = got.double()
         err = (g - w).abs()
         bad = ~_agree(g, w, RTOL, ATOL) & ~self.tainted
+        self.record["values"] += int(w.numel())
         nbad = int(bad.sum())
         rel = torch.nan_to_num(err / (w.abs() + 1e-30), nan=0.0).masked_fill(self.tainted, 0)
         rep.max_rel[name] = float(rel.max()) if rel.numel() else 0.0
@@ -153,15 +180,12 @@ class Lockstep:
         """Local group index of every oracle coordinate."""
         return np.searchsorted(offs, self.idx, side="right") - 1
 
-    def _taint_groups(self, local_js):
-        if not len(local_js):
-            return
-        m = np.zeros(self.d_o, bool)
-        for offs in (self.off_w, self.off_s):
-            gid = self._group_ids(offs)
-            bad_groups = np.unique(gid[local_js])
-            m |= np.isin(gid, bad_groups)
-        self.tainted |= self._dev(m)
+    def _taint(self, local_js):
+        """Exclude these coordinates from later comparisons (their codes differed)."""
+        if len(local_js):
+            m = np.zeros(self.d_o, bool)
+            m[np.asarray(local_js)] = True
+            self.tainted |= self._dev(m)
 
     def _flagged(self, spec, js, u, step, e_old, scale_of, qid, t):
         """Which of the mismatched local coordinates js lie within 2 ulp of a decision threshold."""
@@ -175,7 +199,7 @@ class Lockstep:
                 s = float(scale_of(j))
                 L = 2 ** (spec.bits - 1) - 1
                 y = uj / s * L
-                my = margin * L / s + 2.0 * float(np.spacing(np.float32(abs(y)))) + 4e-7 * abs(y)
+                my = margin * L / s  # the input margin carried to y = u L / s
                 if spec.stochastic:
                     U = O.uniform(self.cfg.seed, qid, t, int(self.idx[j]))
                     fr = y - np.floor(y)
@@ -192,6 +216,12 @@ class Lockstep:
 
     def _compare_codes(self, name, spec, words_view, orc_words, u, step, e_old, scales_orc, offs_local, qid,
                        rep):
+        self.record["code_positions"] += self.d_o
+        if not self.sampled and not bool(self.tainted.any()):
+            # the whole stream at once (padding bits are 0 on both sides); unpacked only if it differs
+            nw = (self.cfg.d * spec.bits + 31) // 32
+            if torch.equal(words_view[:nw], self._dev(orc_words[:nw].view(np.int32))):
+                return
         got = unpack_codes(words_view, self.idx_dev, spec.bits)
         want = unpack_codes(self._dev(orc_words.view(np.int32)), torch.arange(self.d_o, device=self.dev), spec.bits)
         bad = (got != want) & ~self.tainted
@@ -201,15 +231,18 @@ class Lockstep:
             flags = self._flagged(spec, js, u, step, e_old,
                                   (lambda j: scales_orc[gid[j]]) if gid is not None else (lambda j: 0.0),
                                   qid, rep.t - 1)
-            if not flags.all():
-                j = int(js[~flags][0])
-                raise AssertionError(f"round {rep.t}: {name} code differs away from a threshold at local {j} "
-                                     f"(global {int(self.idx[j])}): gpu {int(got[j])} oracle {int(want[j])}, "
-                                     f"u = {float(u[j])!r}")
             rep.code_mismatches += len(js)
             rep.flagged += int(flags.sum())
             self.total_mismatch += len(js)
-            self._taint_groups(js)
+            self.record["mismatches"] += len(js)
+            self.record["flagged"] += int(flags.sum())
+            if self.strict or not flags.all():
+                j = int(js[~flags][0]) if not flags.all() else int(js[0])
+                where = "inside" if flags.all() else "outside"
+                raise AssertionError(f"round {rep.t}: {name}: {len(js)} codes differ ({int(flags.sum())} within 2 ulp "
+                                     f"of a threshold); e.g. local {j} (global {int(self.idx[j])}), {where} the "
+                                     f"window: gpu {int(got[j])} oracle {int(want[j])}, u = {float(u[j])!r}")
+            self._taint(js)
 
     def _compare_scales(self, name, got_view, want, offs_full, rep):
         if not len(want):
@@ -218,22 +251,22 @@ class Lockstep:
             g = got_view.index_select(0, torch.from_numpy(self.groups).to(self.dev))
         else:
             g = got_view[: len(want)]
-        # groups with a tainted coordinate are excluded
-        tainted_groups = []
-        if bool(self.tainted.any()):
-            tainted_groups = np.unique(self._group_ids(offs_full)[self.tainted.cpu().numpy()])
+        self.record["scales"] += len(want)
         w = self._dev(want).double()
         err = ~_agree(g.double(), w, SCALE_RTOL, 0.0)
-        if len(tainted_groups):
-            mask = np.ones(len(want), bool)
-            if self.sampled:
-                mask[np.isin(self.groups, tainted_groups)] = False
-            else:
-                mask[tainted_groups] = False
-            err &= self._dev(mask)
         if bool(err.any()):
-            k = int(torch.nonzero(err)[0])
-            raise AssertionError(f"round {rep.t}: {name} scale {k}: gpu {float(g[k])!r} oracle {float(want[k])!r}")
+            bad = torch.nonzero(err).flatten().cpu().numpy()
+            # a group whose scale differs is accepted only if it holds a coordinate whose code
+            # differed earlier (its l1 / l_inf input then differs); the group is excluded from then on
+            gid = self._group_ids(offs_full)
+            tainted = self.tainted.cpu().numpy()
+            sampled_groups = self.groups if self.sampled else np.arange(len(want))
+            for k in bad:
+                members = gid == sampled_groups[k]
+                if not tainted[members].any():
+                    raise AssertionError(f"round {rep.t}: {name} scale {k}: gpu {float(g[k])!r} "
+                                         f"oracle {float(want[k])!r}")
+                self._taint(np.nonzero(members)[0])
 
     def _compare(self, rep, e_old, es_old, x_dev, x_host):
         cfg, orc, gpu = self.cfg, self.orc, self.gpu

@@ -245,3 +245,37 @@ def test_schedules_follow_the_product_form():
         np.testing.assert_allclose(orc.v[0], v, rtol=4e-7 * t + 1e-6)
         assert np.all(np.abs(orc.m[0] - m) <= (4e-7 * t + 1e-6) * np.max(np.abs(G[: t]), axis=0))
         np.testing.assert_allclose(x, xr, rtol=1e-5, atol=1e-7 * t)
+
+
+@pytest.mark.parametrize("qw,qs", [
+    (W.uniform_q(4, 4096, True), W.uniform_q(8, 4096, False)),
+    (W.sign_q(-1, (9408, 64, 64, 36864, 64, 4096, 5120, 1000)), W.sign_q(-1, (9408, 64, 64, 36864, 64, 4096, 5120,
+                                                                               1000))),
+    (W.pow2_q(-17, -11, 4), W.sign_q(4096)),
+    (W.identity_q(), W.uniform_q(4, 4096, True)),
+])
+@pytest.mark.parametrize("mode", [O.ADAM_AT_WORKER, O.ADAM_AT_SERVER])
+def test_threaded_chunks_equal_one_thread(qw, qs, mode):
+    """The oracle's multi-threaded driver (workers and chunks of whole scale groups on host threads)
+    gives the single-threaded results bit for bit: the chunking only splits separable work."""
+    d = 56_680 if qw.group < 0 else 41_000
+    runs = []
+    for threads in (1, 6):
+        def q(s):
+            offs = O.group_offsets(d, s.group, s.segments if s.group < 0 else None) if s.kind in (1, 2) else \
+                O.group_offsets(d, 0)
+            return O.Quantizer(s.kind, s.bits, offs, s.stochastic, s.pow2_k, s.pow2_K)
+        orc = O.OracleRound(d, 3, q(qw), q(qs), 1e-3, 0.9, 0.999, 1e-8, seed=9, mode=mode, threads=threads)
+        rng = np.random.default_rng(4)
+        x = rng.standard_normal(d).astype(np.float32)
+        for _ in range(3):
+            orc.compress_all([rng.standard_normal(d).astype(np.float32) for _ in range(3)])
+            orc.server_step()
+            orc.apply(x)
+        runs.append((orc, x))
+    (a, xa), (b, xb) = runs
+    assert len(b._chunks) > 1
+    for k in ("e", "m", "v", "es", "ms", "vs", "wwords", "wscales", "swords", "sscales"):
+        assert np.array_equal(getattr(a, k), getattr(b, k)), k
+    assert np.array_equal(xa, xb)
+    assert (a.up_bits, a.down_bits, a.t) == (b.up_bits, b.down_bits, b.t)

@@ -188,7 +188,7 @@ def test_c2_quadratic_toy_full():
     from their own x; ||x - x*|| decreases."""
     w = W.WORKLOADS["c2"]
     cfg = ea.EAConfig.from_workload(w)
-    L = Lockstep(cfg, threads=8)
+    L = Lockstep(cfg)
     xs_host = W.xstar_host(w)
     xs_dev = torch.from_numpy(xs_host).cuda()
     x_dev = torch.zeros(w.d, device="cuda")
@@ -207,45 +207,55 @@ def test_c2_quadratic_toy_full():
     assert all(b < a for a, b in zip(dist[:6], dist[1:7]))
 
 
-def test_c3_resnet18_all_tensors_first_rounds():
+@pytest.mark.parametrize("placement,rounds", [(ea.ADAM_AT_WORKER, 100), (ea.ADAM_AT_SERVER, 10)])
+def test_c3_resnet18_all_tensors(placement, rounds):
+    """All 62 ResNet-18 tensors (per-tensor scales, d = 11,689,512, n = 16) against the full oracle:
+    all 100 rounds in the paper's placement, the first 10 with Adam at the server."""
     w = W.WORKLOADS["c3"]
-    cfg = ea.EAConfig.from_workload(w)
-    L = Lockstep(cfg, threads=16)
+    cfg = ea.EAConfig.from_workload(w, placement=placement)
+    L = Lockstep(cfg)
     x_dev = torch.zeros(w.d, device="cuda")
     x_host = np.zeros(w.d, np.float32)
     bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
-    for t in range(3):
+    for t in range(rounds):
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.total_mismatch == 0
+    if rounds == w.rounds:
+        assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (18_706_393_600, 18_706_393_600)
 
 
-def test_c3_resnet18_sampled_tensors_all_rounds():
-    """All 100 rounds at full size; the oracle follows 14 of the 62 tensors (per-tensor scales make
-    the round separable by tensor), including the smallest, the largest and fc."""
-    w = W.WORKLOADS["c3"]
-    cfg = ea.EAConfig.from_workload(w)
-    groups = [0, 1, 2, 3, 8, 16, 25, 33, 41, 47, 52, 56, 60, 61]
-    L = Lockstep(cfg, sample_groups=groups, threads=16)
-    x_dev = torch.zeros(w.d, device="cuda")
-    x_host = np.zeros(L.d_o, np.float32)
-    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
-    for t in range(w.rounds):
-        _dev_grads(w, t, bufs)
-        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
-    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (18_706_393_600, 18_706_393_600)
-
-
-@pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
-def test_c4_sampled_blocks_all_rounds(placement):
+def test_c4_full_oracle_all_rounds():
+    """c4 (d = 1.1e8, n = 8, 4-bit stochastic / 8-bit grid, 4096-block scales) in the paper's
+    placement against the full oracle: every coordinate of every message and state, all 50 rounds."""
     w = W.WORKLOADS["c4"]
-    cfg = ea.EAConfig.from_workload(w, placement=placement)
-    L = Lockstep(cfg, sample_groups=W.sample_blocks(w, 48), threads=8)
+    cfg = ea.EAConfig.from_workload(w, placement=ea.ADAM_AT_WORKER)
+    L = Lockstep(cfg)
+    x_dev = torch.zeros(w.d, device="cuda")
+    x_host = np.zeros(w.d, np.float32)
+    bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
+    for t in range(w.rounds):
+        _dev_grads(w, t, bufs)
+        L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.total_mismatch == 0
+    assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (176_343_756_800, 352_343_756_800)
+    del L, bufs, x_dev
+    torch.cuda.empty_cache()
+
+
+def test_c4_server_placement_sampled_blocks_all_rounds():
+    """c4 with Adam at the server, all 50 rounds at full size; the oracle follows 1,024 of the
+    26,856 blocks (the round is separable by 4096-block), including the first and the ragged last."""
+    w = W.WORKLOADS["c4"]
+    cfg = ea.EAConfig.from_workload(w, placement=ea.ADAM_AT_SERVER)
+    L = Lockstep(cfg, sample_groups=W.sample_blocks(w, 1024))
     x_dev = torch.zeros(w.d, device="cuda")
     x_host = np.zeros(L.d_o, np.float32)
     bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
     for t in range(w.rounds):
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.total_mismatch == 0
     assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (176_343_756_800, 352_343_756_800)
     del L, bufs, x_dev
     torch.cuda.empty_cache()
@@ -254,16 +264,17 @@ def test_c4_sampled_blocks_all_rounds(placement):
 @pytest.mark.parametrize("placement", [ea.ADAM_AT_WORKER, ea.ADAM_AT_SERVER])
 def test_c5_sampled_blocks_all_rounds(placement):
     """d = 1.558e9, n = 8 on one GPU (W: ~213 GB resident, S: ~126 GB), all 10 rounds; the oracle
-    follows 32 of the 380,372 blocks, including the first and the ragged last one."""
+    follows 1,024 of the 380,372 blocks, including the first and the ragged last one."""
     w = W.WORKLOADS["c5"]
     cfg = ea.EAConfig.from_workload(w, placement=placement)
-    L = Lockstep(cfg, sample_groups=W.sample_blocks(w, 32), threads=8)
+    L = Lockstep(cfg, sample_groups=W.sample_blocks(w, 1024))
     x_dev = torch.zeros(w.d, device="cuda")
     x_host = np.zeros(L.d_o, np.float32)
     bufs = [torch.empty(w.d, device="cuda") for _ in range(w.n)]
     for t in range(w.rounds):
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
+    assert L.total_mismatch == 0
     assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (125_613_752_320, 125_613_752_320)
     del L, bufs, x_dev
     torch.cuda.empty_cache()
