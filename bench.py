@@ -274,18 +274,6 @@ def job_throughput(n: int, d: int, steps: int, world: int, t_max_ms: float) -> f
 NOMINAL_HBM_GBS = 8000.0  # the GB300's nominal ~8 TB/s, the reference of the 70% target
 
 
-def _launches_per_round(w) -> int:
-    """Library kernel launches per round: one per message, plus finalize + encode when the message's
-    scale groups span tiles (the two-pass scale), plus the apply."""
-    from paper_2205_14473_gb300 import workloads as W
-
-    def per_message(spec):
-        has_scale = spec.kind in (W.Q_SIGN_L1, W.Q_UNIFORM_MAX)
-        one_pass = spec.group == 4096 or ((spec.group == 0 or spec.group >= w.d) and w.d <= 4096)
-        return 1 if (not has_scale or one_pass) else 3
-    return w.n * per_message(w.qw) + per_message(w.qs) + 1
-
-
 class RoundTimer:
     """A workload's round state on one device (library handle with its workspace, n resident
     gradients, x) and CUDA-event timing of its rounds on the library's stream."""
@@ -404,6 +392,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int):
     if not args.no_e2e:
         e2e = run_e2e(args, w, rt.rnd, rt.x, dev, stream)
     rnd_ws = rt.rnd.workspace_bytes
+    launches = rt.rnd.launches_per_round
     rt.free()
 
     t_max = max_over_ranks(ms_total, world, dev)
@@ -433,7 +422,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int):
                        "round_gbs": figs["round"]["gbs"],
                        "server_frac_8tbs": figs["server"]["frac_8tbs"],
                        "compress_frac_8tbs": figs["compress"]["frac_8tbs"]},
-        "gpu_launches": _launches_per_round(w) * args.steps,
+        "gpu_launches": launches * args.steps,
         "clocks": clk.summary(),
         "e2e": e2e,
     }
@@ -448,7 +437,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int):
                 ms, c, sv, ap = rte.run(args.extra_steps, max(3, args.warmup), clocks=clk2)
             f = rte.kernel_figures(ms, args.extra_steps, c, sv, ap)
             f["clocks"] = clk2.summary()
-            f["gpu_launches"] = _launches_per_round(we) * args.extra_steps
+            f["gpu_launches"] = rte.rnd.launches_per_round * args.extra_steps
             extra[f"{name}/{'W' if pl == 0 else 'S'}"] = f
             rte.free()
         out["configs"] = extra

@@ -127,6 +127,14 @@ int ea_bits_sent(const ea_handle *h, uint64_t *up_bits, uint64_t *down_bits);
 /* Rounds completed (ea_server_step calls). */
 int ea_round_index(const ea_handle *h, int64_t *t);
 
+/* Kernel launches that one round makes on the stream: n worker compresses, one server step and one
+ * apply.  A message takes one launch, or three when its scale groups span 4096-coordinate tiles
+ * and the one-pass grouped kernel is not used for it: the two-pass scale then adds a finalize and
+ * an encode.  The broadcast takes the grouped kernel whenever its waves fit the device's shared
+ * memory (groups of up to ~7.5 million coordinates on a GB300); the workers' messages only when
+ * the vector has no more 4096-tiles than the grouped kernel has resident CTAs. */
+int ea_round_launches(const ea_handle *h, int32_t *launches);
+
 /* Device views into the workspace (for inspection and checkpoints); index = worker for per-worker
  * views, ignored otherwise.  *bytes receives the view's size.  A view that does not exist in the
  * configured placement returns EA_E_INVAL. */

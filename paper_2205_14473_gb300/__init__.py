@@ -30,7 +30,7 @@ EA_E_CUDA, EA_E_TIMEOUT, EA_E_DEVICE_CHECK, EA_E_UNSUPPORTED = -5, -6, -7, -8
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libea.so")
 EXPORTED = ["ea_workspace_bytes", "ea_init", "ea_worker_compress", "ea_server_step", "ea_worker_apply",
-            "ea_bits_sent", "ea_round_index", "ea_get_view", "ea_sync_status", "ea_last_error", "ea_destroy",
+            "ea_bits_sent", "ea_round_index", "ea_round_launches", "ea_get_view", "ea_sync_status", "ea_last_error", "ea_destroy",
             "ea_worker_compress_noalloc", "ea_set_hparams", "ea_selftest_bounded_wait"]
 
 
@@ -74,6 +74,7 @@ def lib() -> ctypes.CDLL:
             L.ea_worker_apply.argtypes = [_P, _P]
             L.ea_bits_sent.argtypes = [_P, ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_uint64)]
             L.ea_round_index.argtypes = [_P, ctypes.POINTER(ctypes.c_int64)]
+            L.ea_round_launches.argtypes = [_P, ctypes.POINTER(ctypes.c_int32)]
             L.ea_get_view.argtypes = [_P, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_P),
                                       ctypes.POINTER(ctypes.c_size_t)]
             L.ea_sync_status.argtypes = [_P]
@@ -132,6 +133,12 @@ def ea_round_index(h: int) -> int:
     t = ctypes.c_int64(0)
     _check(lib().ea_round_index(h, ctypes.byref(t)), h)
     return t.value
+
+
+def ea_round_launches(h: int) -> int:
+    n = ctypes.c_int32(0)
+    _check(lib().ea_round_launches(h, ctypes.byref(n)), h)
+    return n.value
 
 
 def ea_get_view(h: int, which: int, index: int = 0) -> tuple[int, int]:
@@ -257,6 +264,10 @@ class EARound:
     @property
     def t(self) -> int:
         return ea_round_index(self.h)
+
+    @property
+    def launches_per_round(self) -> int:
+        return ea_round_launches(self.h)
 
     def sync(self) -> None:
         ea_sync_status(self.h)

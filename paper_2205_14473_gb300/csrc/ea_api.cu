@@ -30,16 +30,20 @@ struct QHost {
     bool has_scales = false;
     std::vector<int64_t> offsets;     // GK_SEG
     std::vector<int32_t> tile_group;  // GK_SEG
-    std::vector<int64_t> pair_base;   // PASS_STASH
+    std::vector<int64_t> pair_base;   // PASS_STASH, PASS_GROUPED
+    std::vector<int64_t> cuts;        // PASS_GROUPED: the waves
+    int grid = 0, slots = 0;          // PASS_GROUPED: persistent CTAs and tile slots per CTA
     // device copies (inside the workspace)
-    int64_t *d_offsets = nullptr, *d_pair_base = nullptr;
+    int64_t *d_offsets = nullptr, *d_pair_base = nullptr, *d_cuts = nullptr;
     int32_t *d_tile_group = nullptr;
+    unsigned long long *d_arrive = nullptr;  // PASS_GROUPED: the wave barrier's counter
 };
 
 // Sizes of every workspace buffer, in the order they are carved.
 struct Layout {
     size_t e_w, m_w, v_w, e_s, m_s, v_s, codes_w, scales_w, codes_s, scales_s, partials;
     size_t off_w, tg_w, pb_w, off_s, tg_s, pb_s, status;
+    size_t cuts_w, arr_w, cuts_s, arr_s;  // the grouped pass (groups that span tiles)
     int64_t dpad, wcode_stride, wscale_stride;
 };
 
@@ -59,6 +63,7 @@ struct ea_handle {
     StagePlan splan{};
     Hyper hp{};
     int64_t t = 0;
+    uint64_t epoch_w = 0, epoch_s = 0;  // grouped launches so far (worker messages, broadcasts)
     std::vector<unsigned char> compressed;
     int n_compressed = 0;
     bool has_message = false;
@@ -236,13 +241,20 @@ Layout make_layout(const ea_config &c, const QHost &qw, const QHost &qs)
     L.tg_s = qs.gkind == GK_SEG ? static_cast<size_t>(n_tiles) * 4 : 0;
     L.pb_s = qs.pass == PASS_STASH ? qs.pair_base.size() * 8 : 0;
     L.status = 4;
+    // the grouped pass, whenever groups span tiles (ea_init picks it when its waves fit)
+    const bool gw = qw.pass == PASS_STASH, gs = qs.pass == PASS_STASH;
+    L.cuts_w = gw ? static_cast<size_t>(qw.n_groups + 1) * 8 : 0;
+    L.arr_w = gw ? 8 : 0;
+    L.cuts_s = gs ? static_cast<size_t>(qs.n_groups + 1) * 8 : 0;
+    L.arr_s = gs ? 8 : 0;
     return L;
 }
 
 size_t layout_bytes(const Layout &L)
 {
     const size_t parts[] = {L.e_w, L.m_w, L.v_w, L.e_s, L.m_s, L.v_s, L.codes_w, L.scales_w, L.codes_s,
-                            L.scales_s, L.partials, L.off_w, L.tg_w, L.pb_w, L.off_s, L.tg_s, L.pb_s, L.status};
+                            L.scales_s, L.partials, L.off_w, L.tg_w, L.pb_w, L.off_s, L.tg_s, L.pb_s, L.status,
+                            L.cuts_w, L.arr_w, L.cuts_s, L.arr_s};
     size_t total = 0;
     for (size_t p : parts) total += align_up(p, kAlign);
     return total;
@@ -258,6 +270,84 @@ Grouping device_grouping(const QHost &q)
     g.offsets = q.d_offsets;
     g.tile_group = q.d_tile_group;
     g.pair_base = q.d_pair_base;
+    return g;
+}
+
+// The waves of PASS_GROUPED for q's groups: cuts at group boundaries that start a code word and a
+// float4 slot (multiples of max(4, 32 / b)), each wave touching at most `cap` tiles, greedily as
+// long as possible.  False when some run of groups between two usable cuts needs more tiles.
+bool plan_waves(const QHost &q, int64_t d, int64_t cap, std::vector<int64_t> &cuts)
+{
+    const int64_t align = std::max<int64_t>(4, 32 / q.bits);
+    std::vector<int64_t> cand;
+    if (q.gkind == GK_BLOCK) {
+        for (int64_t b = q.G; b < d; b += q.G)
+            if (b % align == 0) cand.push_back(b);
+    } else if (q.gkind == GK_SEG) {
+        for (size_t i = 1; i + 1 < q.offsets.size(); ++i)
+            if (q.offsets[i] % align == 0) cand.push_back(q.offsets[i]);
+    }
+    cand.push_back(d);
+    auto tiles = [](int64_t a, int64_t b) { return (b - 1) / kTile - a / kTile + 1; };
+    cuts.assign(1, 0);
+    size_t i = 0;
+    for (int64_t c = 0; c < d;) {
+        int64_t best = -1;
+        while (i < cand.size() && tiles(c, cand[i]) <= cap) best = cand[i++];
+        if (best < 0) return false;
+        cuts.push_back(best);
+        c = best;
+    }
+    return true;
+}
+
+// Groups met by one CTA's tile ranges in wave [c0, c1) (tiles t0 + b, t0 + b + grid, ...).
+int64_t cta_groups(const QHost &q, int64_t d, int64_t c0, int64_t c1, int64_t b, int64_t grid)
+{
+    auto group_at = [&](int64_t j) -> int64_t {
+        if (q.gkind == GK_WHOLE) return 0;
+        if (q.gkind == GK_BLOCK) return j / q.G;
+        return std::upper_bound(q.offsets.begin(), q.offsets.end(), j) - q.offsets.begin() - 1;
+    };
+    int64_t total = 0;
+    for (int64_t tile = c0 / kTile + b; tile * kTile < c1; tile += grid) {
+        const int64_t lo = std::max(c0, tile * kTile), hi = std::min({c1, tile * kTile + kTile, d});
+        total += group_at(hi - 1) - group_at(lo) + 1;
+    }
+    return total;
+}
+
+// Switch q from the two-pass scale to the grouped pass if its waves fit this device: `shape` is the
+// grouped kernel's, `sms` the SM count.  max_tiles_per_cta > 0 bounds the tiles each CTA takes
+// (measured on GB300: the grouped worker, whose CTAs run their tiles one after another, is faster
+// than the two passes only while every CTA holds one tile; the grouped server is faster with
+// several).
+void try_grouped(QHost &q, int64_t d, int64_t n_tiles, const GroupedShape &shape, int sms, int max_tiles_per_cta)
+{
+    if (q.pass != PASS_STASH || shape.ctas_per_sm < 1 || shape.slots < 1 || sms < 1) return;
+    const int64_t grid = std::min<int64_t>(static_cast<int64_t>(shape.ctas_per_sm) * sms, n_tiles);
+    const int slots = max_tiles_per_cta > 0 ? std::min(shape.slots, max_tiles_per_cta) : shape.slots;
+    std::vector<int64_t> cuts;
+    if (!plan_waves(q, d, grid * slots, cuts)) return;
+    if (max_tiles_per_cta > 0 && cuts.size() > 2) return;  // one wave only
+    // every CTA's groups of a wave must fit its scale table
+    for (size_t w = 0; w + 1 < cuts.size(); ++w)
+        for (int64_t b = 0; b < grid; ++b)
+            if (cta_groups(q, d, cuts[w], cuts[w + 1], b, grid) > kGroupedScales) return;
+    q.cuts = std::move(cuts);
+    q.grid = static_cast<int>(grid);
+    q.slots = slots;
+    q.pass = PASS_GROUPED;
+}
+
+GroupPlan device_group_plan(const QHost &q, uint64_t epoch)
+{
+    GroupPlan g{};
+    g.n_waves = static_cast<int64_t>(q.cuts.size()) - 1;
+    g.cuts = q.d_cuts;
+    g.arrive = q.d_arrive;
+    g.epoch = epoch;
+    g.slots = q.slots;
     return g;
 }
 
@@ -397,6 +487,25 @@ cudaError_t ea::launch_server(int mode, const ServerArgs &a, cudaStream_t s)
     }
 }
 
+cudaError_t ea::launch_server_grouped(int mode, const ServerArgs &a, int grid, cudaStream_t s)
+{
+    if (mode == MODE_W)
+        return a.qs.kind == QK_SIGN ? launch_server_grouped_for_qs<MODE_W, QK_SIGN>(a, grid, s)
+                                    : launch_server_grouped_for_qs<MODE_W, QK_UNIF>(a, grid, s);
+    return a.qs.kind == QK_SIGN ? launch_server_grouped_for_qs<MODE_S, QK_SIGN>(a, grid, s)
+                                : launch_server_grouped_for_qs<MODE_S, QK_UNIF>(a, grid, s);
+}
+
+cudaError_t ea::server_grouped_shape(int mode, int qw, int qs, GroupedShape *out)
+{
+    if (qs != QK_SIGN && qs != QK_UNIF) return cudaErrorNotSupported;
+    if (mode == MODE_W)
+        return qs == QK_SIGN ? server_grouped_shape_for_qs<MODE_W, QK_SIGN>(qw, out)
+                             : server_grouped_shape_for_qs<MODE_W, QK_UNIF>(qw, out);
+    return qs == QK_SIGN ? server_grouped_shape_for_qs<MODE_S, QK_SIGN>(qw, out)
+                         : server_grouped_shape_for_qs<MODE_S, QK_UNIF>(qw, out);
+}
+
 extern "C" {
 
 int ea_workspace_bytes(const ea_config *cfg, size_t *bytes)
@@ -467,10 +576,25 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->qs.d_tile_group = reinterpret_cast<int32_t *>(take(L.tg_s));
     h->qs.d_pair_base = reinterpret_cast<int64_t *>(take(L.pb_s));
     h->status = reinterpret_cast<uint32_t *>(take(L.status));
+    h->qw.d_cuts = reinterpret_cast<int64_t *>(take(L.cuts_w));
+    h->qw.d_arrive = reinterpret_cast<unsigned long long *>(take(L.arr_w));
+    h->qs.d_cuts = reinterpret_cast<int64_t *>(take(L.cuts_s));
+    h->qs.d_arrive = reinterpret_cast<unsigned long long *>(take(L.arr_s));
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) == cudaSuccess &&
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess) {
         h->splan = make_server_plan(*cfg, h->qw, h->qs, h->n_tiles, sms);
+        // groups that span tiles: the one-pass grouped kernels when their waves fit, else two passes
+        const int mode = cfg->placement == EA_ADAM_AT_WORKER ? MODE_W : MODE_S;
+        int coop = 0;
+        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+        GroupedShape shw{}, shs{};
+        if (coop && h->qw.pass == PASS_STASH && worker_grouped_shape(mode, h->qw.kind, &shw) == cudaSuccess)
+            try_grouped(h->qw, cfg->d, h->n_tiles, shw, sms, 1);
+        if (coop && h->qs.pass == PASS_STASH && server_grouped_shape(mode, h->qw.kind, h->qs.kind, &shs) == cudaSuccess)
+            try_grouped(h->qs, cfg->d, h->n_tiles, shs, sms, 0);
+        cudaGetLastError();  // a shape query that failed leaves the two-pass scale in place
+    }
 
     // Algorithm 2: m_0 = 0, v_0 = eps (0 in the textbook form), e_1 = 0; Algorithm 1: e_1 = 0.
     // Messages start zeroed.
@@ -490,6 +614,8 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     upload(h->qs.d_offsets, h->qs.offsets.data(), L.off_s);
     upload(h->qs.d_tile_group, h->qs.tile_group.data(), L.tg_s);
     upload(h->qs.d_pair_base, h->qs.pair_base.data(), L.pb_s);
+    upload(h->qw.d_cuts, h->qw.cuts.data(), h->qw.cuts.size() * 8);
+    upload(h->qs.d_cuts, h->qs.cuts.data(), h->qs.cuts.size() * 8);
     if (r != EA_OK) {
         g_last_error = h->err;
         delete h;
@@ -526,7 +652,14 @@ int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
     a.id = static_cast<uint32_t>(worker);
     a.t = static_cast<uint32_t>(h->t);
     a.partials = h->partials;
-    r = check_cuda(h, launch_worker(W ? MODE_W : MODE_S, a, h->stream), "worker launch");
+    a.status = h->status;
+    if (h->qw.pass == PASS_GROUPED) {
+        a.gp = device_group_plan(h->qw, h->epoch_w);
+        r = check_cuda(h, launch_worker_grouped(W ? MODE_W : MODE_S, a, h->qw.grid, h->stream), "worker launch");
+        if (r == EA_OK) ++h->epoch_w;
+    } else {
+        r = check_cuda(h, launch_worker(W ? MODE_W : MODE_S, a, h->stream), "worker launch");
+    }
     if (r == EA_OK && h->qw.pass == PASS_STASH) r = second_pass(h, h->qw, a.e, a.words, a.scales, a.id);
     if (r != EA_OK) return r;
     h->compressed[worker] = 1;
@@ -566,7 +699,14 @@ int ea_server_step(ea_handle *h)
     a.status = h->status;
     a.plan = h->splan;
     const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
-    int r = check_cuda(h, launch_server(W ? MODE_W : MODE_S, a, h->stream), "server launch");
+    int r;
+    if (h->qs.pass == PASS_GROUPED) {
+        a.gp = device_group_plan(h->qs, h->epoch_s);
+        r = check_cuda(h, launch_server_grouped(W ? MODE_W : MODE_S, a, h->qs.grid, h->stream), "server launch");
+        if (r == EA_OK) ++h->epoch_s;
+    } else {
+        r = check_cuda(h, launch_server(W ? MODE_W : MODE_S, a, h->stream), "server launch");
+    }
     if (r == EA_OK && h->qs.pass == PASS_STASH)
         r = second_pass(h, h->qs, h->es, h->scodes, h->sscales, static_cast<uint32_t>(h->cfg.n));
     if (r != EA_OK) return r;
@@ -615,6 +755,14 @@ int ea_bits_sent(const ea_handle *h, uint64_t *up_bits, uint64_t *down_bits)
     if (!h || !up_bits || !down_bits) return fail(nullptr, EA_E_INVAL, "NULL argument");
     *up_bits = h->up_bits;
     *down_bits = h->down_bits;
+    return EA_OK;
+}
+
+int ea_round_launches(const ea_handle *h, int32_t *launches)
+{
+    if (!h || !launches) return fail(nullptr, EA_E_INVAL, "NULL argument");
+    auto per_message = [](const QHost &q) { return q.pass == PASS_STASH ? 3 : 1; };
+    *launches = h->cfg.n * per_message(h->qw) + per_message(h->qs) + 1;
     return EA_OK;
 }
 

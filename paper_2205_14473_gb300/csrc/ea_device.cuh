@@ -290,6 +290,8 @@ __device__ __forceinline__ int code_bits(const QParams &q)
 }
 
 // ----------------------------------------------------------------------------- scale groups
+// (The lookups below read the segment offsets from global memory one by one; per-coordinate
+// lookups on tiles that hold several segments go through TileGroups instead.)
 
 __device__ __forceinline__ int64_t group_begin(const Grouping &g, int64_t gi, int64_t d)
 {
@@ -337,6 +339,48 @@ __device__ __forceinline__ int64_t tile_single_group(const Grouping &g, int64_t 
     return g.offsets[g0 + 1] > last ? g0 : -1;
 }
 
+// The segments (GK_SEG) of one tile, for per-coordinate lookups from shared memory: the tile's
+// first group and the offsets, from the tile's start, of the groups that start inside it.
+constexpr int kTileBounds = 64;
+struct TileGroups {
+    int64_t g0;
+    int nb;                          // groups starting inside the tile; > kTileBounds: not cached
+    uint16_t b[kTileBounds];
+};
+
+// Fill tg for tile `tile` (all threads; the caller puts a barrier between this and the lookups).
+__device__ __forceinline__ void cache_tile_groups(const Grouping &g, int64_t tile, int64_t d, TileGroups &tg)
+{
+    const int64_t tl = tile * kTile;
+    const int64_t n_tiles = (d + kTile - 1) / kTile;
+    const int64_t g0 = g.tile_group[tile];
+    int64_t last;  // the group holding the tile's last coordinate
+    if (tile + 1 < n_tiles) {
+        const int64_t gn = g.tile_group[tile + 1];
+        last = g.offsets[gn] == tl + kTile ? gn - 1 : gn;
+    } else {
+        last = g.n_groups - 1;
+    }
+    const int nb = static_cast<int>(last - g0);
+    if (threadIdx.x == 0) {
+        tg.g0 = g0;
+        tg.nb = nb;
+    }
+    if (nb <= kTileBounds)
+        for (int i = threadIdx.x; i < nb; i += blockDim.x)
+            tg.b[i] = static_cast<uint16_t>(g.offsets[g0 + 1 + i] - tl);
+}
+
+// Group of coordinate j of the cached tile (falls back to the global scan past kTileBounds groups).
+__device__ __forceinline__ int64_t tile_group_of(const Grouping &g, const TileGroups &tg, int64_t tile, int64_t j)
+{
+    if (tg.nb > kTileBounds) return group_of(g, j, tg.g0);
+    const uint32_t x = static_cast<uint32_t>(j - tile * kTile);
+    int c = 0;
+    for (int i = 0; i < tg.nb; ++i) c += tg.b[i] <= x ? 1 : 0;
+    return tg.g0 + c;
+}
+
 // --------------------------------------------------------------------------------- packing
 // Coordinate j's b-bit code sits at bit j*b of the little-endian word stream.  A float4 slot q
 // (coordinates 4q .. 4q+3) spans 4b bits, so for b <= 8 it lies inside word (q*b)/8.
@@ -376,14 +420,16 @@ __device__ __forceinline__ uint32_t spread8_by4(uint32_t x)
 }
 
 // Store the four codes of slot q (the same slot index on every lane is q_lane0 + lane).  Must be
-// called by all 32 lanes of the warp.  Codes of coordinates >= d are 0 (caller's job).
+// called by all 32 lanes of the warp.  Only words whose first coordinate lies in [lo, hi) are
+// written (lo starts a word; codes of coordinates >= hi are 0, the caller's job), so that two
+// ranges that meet at a word boundary never write the same word.
 // b = 1: one ballot per component; lanes 8g .. 8g+7 fill word (q_lane0 / 8) + g, whose bit
 // 4l + c is component c of lane 8g + l.
 // b in {2, 4, 8}: the slot's 4b bits, shifted to its place in the word and OR-ed across the 8/b
 // lanes that share the word (compile-time width).
 template <int B, bool FULL>
 __device__ __forceinline__ void store_codes4_narrow(uint32_t *__restrict__ words, int64_t q, const uint32_t c[4],
-                                                    int64_t n_words)
+                                                    int64_t lo, int64_t hi)
 {
     constexpr int per_word = 8 / B;  // slots per word: 4 (b=2), 2 (b=4), 1 (b=8)
     uint32_t v = c[0] | (c[1] << B) | (c[2] << (2 * B)) | (c[3] << (3 * B));
@@ -392,12 +438,13 @@ __device__ __forceinline__ void store_codes4_narrow(uint32_t *__restrict__ words
     if (per_word >= 2) v |= __shfl_xor_sync(0xffffffffu, v, 1);
     if (per_word >= 4) v |= __shfl_xor_sync(0xffffffffu, v, 2);
     const int64_t wi = (q * B) >> 3;
-    if (pos == 0 && (FULL || wi < n_words)) words[wi] = v;
+    const int64_t first = 4 * q;  // pos == 0: the word's first coordinate
+    if (pos == 0 && (FULL || (first >= lo && first < hi))) words[wi] = v;
 }
 
 template <bool FULL = false, bool BALLOT = true>
 __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64_t q, int bits, const uint32_t c[4],
-                                             int64_t n_words)
+                                             int64_t lo, int64_t hi)
 {
     const int lane = threadIdx.x & 31;
     if (bits == 1 && !BALLOT) {
@@ -407,7 +454,7 @@ __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64
         v |= __shfl_xor_sync(0xffffffffu, v, 2);
         v |= __shfl_xor_sync(0xffffffffu, v, 4);
         const int64_t wi = q >> 3;
-        if ((lane & 7) == 0 && (FULL || wi < n_words)) words[wi] = v;
+        if ((lane & 7) == 0 && (FULL || (32 * wi >= lo && 32 * wi < hi))) words[wi] = v;
     } else if (bits == 1) {
         const uint32_t b0 = __ballot_sync(0xffffffffu, c[0] != 0);
         const uint32_t b1 = __ballot_sync(0xffffffffu, c[1] != 0);
@@ -418,19 +465,20 @@ __device__ __forceinline__ void store_codes4(uint32_t *__restrict__ words, int64
             const uint32_t w = spread8_by4(b0 >> sh) | (spread8_by4(b1 >> sh) << 1) | (spread8_by4(b2 >> sh) << 2) |
                                (spread8_by4(b3 >> sh) << 3);
             const int64_t wi = ((q - lane) >> 3) + lane;  // q - lane is lane 0's slot
-            if (FULL || wi < n_words) words[wi] = w;
+            if (FULL || (32 * wi >= lo && 32 * wi < hi)) words[wi] = w;
         }
     } else if (bits == 2) {
-        store_codes4_narrow<2, FULL>(words, q, c, n_words);
+        store_codes4_narrow<2, FULL>(words, q, c, lo, hi);
     } else if (bits == 4) {
-        store_codes4_narrow<4, FULL>(words, q, c, n_words);
+        store_codes4_narrow<4, FULL>(words, q, c, lo, hi);
     } else if (bits == 8) {
-        store_codes4_narrow<8, FULL>(words, q, c, n_words);
+        store_codes4_narrow<8, FULL>(words, q, c, lo, hi);
     } else if (bits == 16) {
-        if (FULL || 2 * q < n_words)
+        if (FULL || (4 * q >= lo && 4 * q < hi))
             reinterpret_cast<uint2 *>(words)[q] = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
     } else {
-        if (FULL || 4 * q < n_words) reinterpret_cast<uint4 *>(words)[q] = make_uint4(c[0], c[1], c[2], c[3]);
+        if (FULL || (4 * q >= lo && 4 * q < hi))
+            reinterpret_cast<uint4 *>(words)[q] = make_uint4(c[0], c[1], c[2], c[3]);
     }
 }
 

@@ -68,9 +68,36 @@ inline float bias_correction(float beta, int64_t t1)
 
 // How the scale of a message is formed.
 enum Pass : int {
-    PASS_FUSED = 0,  // every group lies inside one tile: reduce, encode and store in one pass
-    PASS_STASH = 1   // groups span tiles: store the input in the residual buffer plus one
-                     // partial norm per (tile, group); finalize_kernel and encode_kernel finish
+    PASS_FUSED = 0,   // every group lies inside one tile: reduce, encode and store in one pass
+    PASS_STASH = 1,   // groups span tiles: store the input in the residual buffer plus one
+                      // partial norm per (tile, group); finalize_kernel and encode_kernel finish
+    PASS_GROUPED = 2  // groups span tiles, one cooperative pass: the input stays in shared memory
+                      // while the group's partial norms are combined (GroupPlan)
+};
+
+// The one-pass plan for scale groups that span tiles.  The vector is cut into waves, coordinate
+// ranges [cuts[w], cuts[w+1]) of whole groups whose tiles fit in shared memory at once (every cut
+// starts a code word and a float4 slot).  A persistent CTA takes the wave's tiles blockIdx.x,
+// blockIdx.x + gridDim.x, ... (at most `slots`), parks each tile's input in shared memory and
+// stores one partial norm per (group, tile); after a grid-wide barrier every CTA combines, in a
+// fixed order, the partials of the groups its tiles need, and encodes its tiles.  The launch is
+// cooperative (all CTAs resident), so the barrier completes; its wait is still bounded and
+// reports EA_E_TIMEOUT.
+struct GroupPlan {
+    int64_t n_waves;
+    const int64_t *cuts;         // n_waves + 1 coordinate offsets (device)
+    unsigned long long *arrive;  // CTAs arrived at the wave barriers, over all launches
+    uint64_t epoch;              // launches made with this counter before this one
+    int slots;                   // tiles of input a CTA holds in shared memory
+};
+
+// Scales of groups a grouped CTA holds in shared memory for one wave (the plan keeps the grouped
+// pass off when some CTA's tiles of a wave meet more groups).
+constexpr int kGroupedScales = 256;
+
+// Shape of a grouped kernel on this device: CTAs per SM and tile slots per CTA.
+struct GroupedShape {
+    int ctas_per_sm, slots;
 };
 
 struct WorkerArgs {
@@ -85,6 +112,8 @@ struct WorkerArgs {
     uint64_t seed;
     uint32_t id, t;
     double *partials;
+    GroupPlan gp;             // PASS_GROUPED
+    uint32_t *status;         // device status word (timeouts); may be null outside a handle
 };
 
 // Shared-memory staging plan of the pipelined (persistent, bulk-copy) kernels.  A stage holds one
@@ -121,6 +150,7 @@ struct ServerArgs {
     int64_t wcode_bytes;      // padded bytes of one worker's code stream (multiple of 256)
     uint32_t *status;         // device status word (timeouts)
     StagePlan plan;
+    GroupPlan gp;             // PASS_GROUPED (Q_s's groups)
 };
 
 // Second pass of PASS_STASH: encode the stashed input in buf, leave the residual in buf.
@@ -151,6 +181,15 @@ struct ApplyArgs {
 };
 
 cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s);
+// The one-pass kernels of PASS_GROUPED (cooperative launches of `grid` CTAs) and their shapes.
+cudaError_t launch_worker_grouped(int mode, const WorkerArgs &a, int grid, cudaStream_t s);
+cudaError_t worker_grouped_shape(int mode, int qk, GroupedShape *out);
+template <int MODE, int QS>
+cudaError_t launch_server_grouped_for_qs(const ServerArgs &a, int grid, cudaStream_t s);
+template <int MODE, int QS>
+cudaError_t server_grouped_shape_for_qs(int qw, GroupedShape *out);
+cudaError_t launch_server_grouped(int mode, const ServerArgs &a, int grid, cudaStream_t s);
+cudaError_t server_grouped_shape(int mode, int qw, int qs, GroupedShape *out);
 // The server kernel for one placement and broadcast quantizer kind; each (MODE, QS) pair is
 // instantiated only in its own translation unit, ea_server_<mode>_q<QS>.cu.
 template <int MODE, int QS>

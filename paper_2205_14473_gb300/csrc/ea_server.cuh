@@ -4,52 +4,28 @@
 #include <atomic>
 
 #include "ea_async.cuh"
+#include "ea_grouped.cuh"
 #include "ea_tile.cuh"
 
 namespace ea {
 
-// Decode the n worker messages of this tile, average them (summed in worker order, one division
-// by n), add the server residual (and, with Adam at the server, take the Adam step on the
-// average first), then Q_s and e_s <- w - Q_s(w) (finish_tile).
-// HBM traffic per coordinate: n b_w/8 B of worker codes + 4 B e_s read + 4 B e_s written + b_s/8 B
-// of broadcast code (+ 16 B for m, v with Adam at the server).
-template <int MODE, int QW, int QS>
-__global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
+// The worker-order sum of the n decoded worker messages at this thread's 16 coordinates of tile
+// `tile` (coordinates >= d give 0), read straight from global memory.  utab: fl(i / L) of the
+// workers' uniform grid (b_w <= 8) or null; stab: 256 floats of shared memory for the sign table.
+// Contains a CTA barrier (all threads call it; the caller orders stab's previous readers before it).
+template <int QW>
+__device__ __forceinline__ void decode_sum_direct(const ServerArgs &a, int64_t tile, const float *utab, float *stab,
+                                                  TileGroups &tg, float (&acc)[kSlots][4])
 {
-    __shared__ TileSmem sm;
-    __shared__ float utab[256];  // fl(i / L) for the workers' uniform grid, i = -L..L (b_w <= 8)
-    const int64_t tile = blockIdx.x;
     const int64_t d = a.d;
-
     const int Lw = (QW == QK_UNIF) ? unif_L(a.qw.bits) : 0;
     const float Lwf = static_cast<float>(Lw);
-    const bool use_tab = QW == QK_UNIF && a.qw.bits <= 8;
-    build_qtab<QS>(a.qs, sm.qtab);  // read after the scale reduction's barrier
-    if (use_tab) {
-        for (int i = threadIdx.x; i <= 2 * Lw; i += kThreads)
-            utab[i] = __fdiv_rn(static_cast<float>(i - Lw), Lwf);
-        __syncthreads();
-    }
-
-    float es[kSlots][4], ms[kSlots][4], vs[kSlots][4];
-#pragma unroll
-    for (int k = 0; k < kSlots; ++k) {
-        const int64_t q = slot_of(tile, k);
-        load4(a.es, q, d, es[k]);
-        if (MODE == MODE_S) {
-            load4(a.ms, q, d, ms[k]);
-            load4(a.vs, q, d, vs[k]);
-        }
-    }
-
     // The workers' scale of a coordinate: one per worker for the whole tile when the tile lies
     // in one of Q_w's groups (always for 4096-blocks), else a per-coordinate group lookup.
     const Grouping &GW = a.qw.grp;
     const int64_t wg = has_scale<QW>() ? tile_single_group(GW, tile, d) : 0;
     const bool wtile = wg >= 0;
     const int64_t whint = first_group_of_tile(GW, tile);
-
-    float acc[kSlots][4];
 #pragma unroll
     for (int k = 0; k < kSlots; ++k)
 #pragma unroll
@@ -63,7 +39,6 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
     // remaining workers are then added in order.
     int w_first = 0;
     if constexpr (QW == QK_SIGN) {
-        __shared__ float stab[256];
         if (wtile) {
             const int m = min(a.n, 8);
             constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
@@ -94,6 +69,27 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
         }
     }
 
+    // a tile over several groups: each coordinate's group, looked up once (segments from shared
+    // memory), as an offset from the tile's first group (a tile of 4096 coordinates meets at most
+    // 4096 groups: 16 bits per coordinate)
+    const bool seg = has_scale<QW>() && !wtile && GW.gkind == GK_SEG;
+    if (seg) {
+        cache_tile_groups(GW, tile, d, tg);
+        __syncthreads();
+    }
+    uint32_t gl[kSlots][2] = {{0u, 0u}, {0u, 0u}, {0u, 0u}, {0u, 0u}};
+    if (has_scale<QW>() && !wtile) {
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            const int64_t j0 = 4 * slot_of(tile, k);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int64_t j = j0 + i < d ? j0 + i : d - 1;
+                const int64_t g = (seg ? tile_group_of(GW, tg, tile, j) : group_of(GW, j, whint)) - whint;
+                gl[k][i >> 1] |= static_cast<uint32_t>(g) << (16 * (i & 1));
+            }
+        }
+    }
 #pragma unroll 2
     for (int w = w_first; w < a.n; ++w) {
         const uint32_t *ww = a.wwords + static_cast<int64_t>(w) * a.wwords_stride;
@@ -110,12 +106,57 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
             for (int i = 0; i < 4; ++i) {
                 if (j0 + i < d) {
                     float s = 0.0f;
-                    if (has_scale<QW>()) s = wtile ? s_tile : __ldg(wsc + group_of(GW, j0 + i, whint));
-                    acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], s, a.qw, Lwf, Lw, use_tab ? utab : nullptr));
+                    if (has_scale<QW>())
+                        s = wtile ? s_tile : __ldg(wsc + whint + ((gl[k][i >> 1] >> (16 * (i & 1))) & 0xffffu));
+                    acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], s, a.qw, Lwf, Lw, utab));
                 }
             }
         }
     }
+}
+
+// The workers' uniform grid's fl(i / L), i = -L .. L, into utab (b_w <= 8; no barrier).
+template <int QW>
+__device__ __forceinline__ const float *build_worker_utab(const ServerArgs &a, float *utab)
+{
+    if (QW != QK_UNIF || a.qw.bits > 8) return nullptr;
+    const int Lw = unif_L(a.qw.bits);
+    for (int i = threadIdx.x; i <= 2 * Lw; i += blockDim.x)
+        utab[i] = __fdiv_rn(static_cast<float>(i - Lw), static_cast<float>(Lw));
+    return utab;
+}
+
+// Decode the n worker messages of this tile, average them (summed in worker order, one division
+// by n), add the server residual (and, with Adam at the server, take the Adam step on the
+// average first), then Q_s and e_s <- w - Q_s(w) (finish_tile).
+// HBM traffic per coordinate: n b_w/8 B of worker codes + 4 B e_s read + 4 B e_s written + b_s/8 B
+// of broadcast code (+ 16 B for m, v with Adam at the server).
+template <int MODE, int QW, int QS>
+__global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
+{
+    __shared__ TileSmem sm;
+    __shared__ float utab_s[256];  // fl(i / L) for the workers' uniform grid, i = -L..L (b_w <= 8)
+    __shared__ float stab[256];
+    __shared__ TileGroups tg;
+    const int64_t tile = blockIdx.x;
+    const int64_t d = a.d;
+
+    build_qtab<QS>(a.qs, sm.qtab);  // read after the scale reduction's barrier
+    const float *utab = build_worker_utab<QW>(a, utab_s);
+    if (utab) __syncthreads();
+
+    float es[kSlots][4], ms[kSlots][4], vs[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        load4(a.es, q, d, es[k]);
+        if (MODE == MODE_S) {
+            load4(a.ms, q, d, ms[k]);
+            load4(a.vs, q, d, vs[k]);
+        }
+    }
+    float acc[kSlots][4];
+    decode_sum_direct<QW>(a, tile, utab, stab, tg, acc);
 
     const float nf = static_cast<float>(a.n);
     const bool pow2n = (a.n & (a.n - 1)) == 0;
@@ -140,17 +181,43 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
                     static_cast<uint32_t>(a.n), a.t, a.partials, sm);
 }
 
-
-constexpr int kWorkerTab = 1024;  // floats of the staged server's per-tile worker table
-
-// Bits 0, 4, ..., 28 of x moved to bits 0 .. 7 (the inverse of spread8_by4).
-__device__ __forceinline__ uint32_t gather_every4(uint32_t x)
+// Phase one of a grouped server tile: w (the average, after the Adam step with Adam at the server,
+// plus e_s) of the coordinate range [lo, hi) of tile `tile` (0 elsewhere) into ub; m_s and v_s
+// updated and stored in the range.  FULL: the range is the whole tile.
+template <int MODE, int QW, bool FULL>
+__device__ __forceinline__ void server_u_range(const ServerArgs &a, int64_t tile, int64_t lo, int64_t hi, float4 *ub,
+                                               const float *utab, float *stab, TileGroups &tg)
 {
-    x &= 0x11111111u;
-    x = (x | (x >> 3)) & 0x03030303u;
-    x = (x | (x >> 6)) & 0x000f000fu;
-    x = (x | (x >> 12)) & 0x000000ffu;
-    return x;
+    float acc[kSlots][4];
+    decode_sum_direct<QW>(a, tile, utab, stab, tg, acc);
+    const float nf = static_cast<float>(a.n);
+    const bool pow2n = (a.n & (a.n - 1)) == 0;
+    const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        const int64_t j0 = 4 * q;
+        const bool in = FULL || (j0 >= lo && j0 < hi);
+        float es[4] = {0.f, 0.f, 0.f, 0.f}, ms[4] = {0.f, 0.f, 0.f, 0.f}, vs[4] = {1.f, 1.f, 1.f, 1.f}, u[4];
+        if (in) {
+            load4<FULL>(a.es, q, hi, es);
+            if (MODE == MODE_S) {
+                load4<FULL>(a.ms, q, hi, ms);
+                load4<FULL>(a.vs, q, hi, vs);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float step = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
+            if (MODE == MODE_S) step = adam_step(step, ms[i], vs[i], a.hp);
+            u[i] = (in && (FULL || j0 + i < hi)) ? __fadd_rn(step, es[i]) : 0.0f;
+        }
+        ub[k * kThreads + threadIdx.x] = make_float4(u[0], u[1], u[2], u[3]);
+        if (MODE == MODE_S && in) {
+            store4<FULL>(a.ms, q, hi, ms);
+            store4<FULL>(a.vs, q, hi, vs);
+        }
+    }
 }
 
 // Load the four codes of local slot ls (0 .. 1023) of a tile's code chunk held in shared memory.
@@ -175,6 +242,236 @@ __device__ __forceinline__ void load_codes4_smem(const uint32_t *words, int ls, 
         c[2] = w.z;
         c[3] = w.w;
     }
+}
+
+constexpr int kWorkerScales = 512;  // worker scales of a tile's groups held by the grouped server
+
+// Whether the grouped server stages a tile's worker codes in shared memory: all n chunks must fit
+// in the tile's slot (4096 b_w / 8 bytes each, 16 KB in all).
+__device__ __forceinline__ bool server_codes_fit(const ServerArgs &a, int bw) { return a.n * bw <= 32; }
+
+// The worker-order sum of the n decoded worker messages at this thread's 16 coordinates of tile
+// `tile`, from the tile's code chunks staged in shared memory (cw: worker w's chunk at
+// w * chunk_words) and the workers' scales of the tile's groups (wsc: worker w's scale of the
+// tile's group gw0 + g at w * ngw + g).  seg: the tile holds several of Q_w's segments (tg holds
+// them); ngw > 1 without seg: several blocks (looked up arithmetically).  Contains a CTA barrier.
+template <int QW>
+__device__ __forceinline__ void decode_sum_staged(const ServerArgs &a, int64_t tile, const uint32_t *cw,
+                                                  int chunk_words, const float *wsc, int ngw, int64_t gw0, bool seg,
+                                                  const TileGroups &tg, float *stab, const float *utab,
+                                                  float (&acc)[kSlots][4])
+{
+    const int n = a.n;
+    const int bw = code_bits<QW>(a.qw);
+    const int Lw = (QW == QK_UNIF) ? unif_L(a.qw.bits) : 0;
+    const float Lwf = static_cast<float>(Lw);
+    const Grouping &GW = a.qw.grp;
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[k][i] = 0.0f;
+    int w_first = 0;
+    if constexpr (QW == QK_SIGN) {
+        if (ngw == 1) {
+            // the worker-order sum of the first m = min(n, 8) workers by sign pattern (worker w's
+            // code at bit pi(w), pi = (0, 4, 1, 5, 2, 6, 3, 7)), thread p forming pattern p's sum as
+            // the loop below would
+            const int m = min(n, 8);
+            constexpr uint32_t pi = 0x73625140u;  // pi(w) in nibble w
+            float t = 0.0f;
+            for (int w = 0; w < m; ++w)
+                t = __fadd_rn(t, ((threadIdx.x >> ((pi >> (4 * w)) & 7u)) & 1u) ? wsc[w] : -wsc[w]);
+            stab[threadIdx.x] = t;
+            compute_sync();
+            const int sh = 4 * (threadIdx.x & 7);  // this thread's nibble in every code word
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k) {
+                const int ls = k * kThreads + threadIdx.x;
+                uint32_t X = 0;  // bit 4w + i: worker w's code of the slot's coordinate i
+#pragma unroll
+                for (int w = 0; w < 8; ++w)
+                    if (w < m) X |= ((cw[w * chunk_words + (ls >> 3)] >> sh) & 0xfu) << (4 * w);
+                // bits 4w of X >> i times 0x01020408 land, without carries, at 24 + pi(w)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[k][i] = stab[(((X >> i) & 0x11111111u) * 0x01020408u) >> 24];
+            }
+            w_first = m;
+        }
+    }
+    // each coordinate's group within the tile (0 .. ngw - 1 <= 255: the caller's table bound),
+    // looked up once, one byte per coordinate of a slot
+    uint32_t gl[kSlots] = {0u, 0u, 0u, 0u};
+    if (has_scale<QW>() && ngw > 1) {
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            const int64_t j0 = 4 * slot_of(tile, k);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int64_t j = j0 + i < a.d ? j0 + i : a.d - 1;
+                const int64_t g = (seg ? tile_group_of(GW, tg, tile, j) : group_of(GW, j, gw0)) - gw0;
+                gl[k] |= static_cast<uint32_t>(g) << (8 * i);
+            }
+        }
+    }
+#pragma unroll 1
+    for (int w = w_first; w < n; ++w) {
+        const uint32_t *ww = cw + w * chunk_words;
+        const float *ws = wsc + w * ngw;
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            const int ls = k * kThreads + threadIdx.x;
+            uint32_t c[4];
+            load_codes4_smem(ww, ls, bw, c);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float s = has_scale<QW>() ? ws[(gl[k] >> (8 * i)) & 0xffu] : 0.0f;
+                acc[k][i] = __fadd_rn(acc[k][i], decode1<QW>(c[i], s, a.qw, Lwf, Lw, utab));
+            }
+        }
+    }
+}
+
+// Phase one of a grouped server tile, inputs staged in shared memory: the tile's worker code
+// chunks go into the tile's own slot ub (free until w lands in it) and the workers' scales of its
+// groups into wsc, all loads issued at once; then the decode reads shared memory only.  w (the
+// average, after the Adam step with Adam at the server, plus e_s) of the range [lo, hi) then
+// replaces the codes in ub (0 outside the range); m_s, v_s are updated and stored in the range.
+// Returns false, having done nothing, when the tile's scale table would not fit (the caller then
+// takes server_u_range).
+template <int MODE, int QW, bool FULL>
+__device__ __forceinline__ bool server_u_staged(const ServerArgs &a, int64_t tile, int64_t lo, int64_t hi, float4 *ub,
+                                                const float *utab, float *stab, float *wsc, GroupSmem &gs)
+{
+    const int64_t d = a.d;
+    const int n = a.n;
+    const int bw = code_bits<QW>(a.qw);
+    const Grouping &GW = a.qw.grp;
+    int64_t gw0 = 0;
+    int ngw = 1;
+    if (has_scale<QW>()) {
+        gw0 = first_group_of_tile(GW, tile);
+        const int64_t last = min(tile * kTile + static_cast<int64_t>(kTile), d) - 1;
+        ngw = static_cast<int>(group_of(GW, last, gw0) - gw0 + 1);
+        if (n * ngw > kWorkerScales || ngw > 256) return false;
+    }
+    const bool seg = has_scale<QW>() && ngw > 1 && GW.gkind == GK_SEG;
+    float es[kSlots][4], ms[kSlots][4], vs[kSlots][4];
+    bool in[kSlots];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        in[k] = FULL || (4 * q >= lo && 4 * q < hi);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) es[k][i] = ms[k][i] = 0.0f, vs[k][i] = 1.0f;
+        if (in[k]) {
+            load4<FULL>(a.es, q, hi, es[k]);
+            if (MODE == MODE_S) {
+                load4<FULL>(a.ms, q, hi, ms[k]);
+                load4<FULL>(a.vs, q, hi, vs[k]);
+            }
+        }
+    }
+    compute_sync();  // the slot's and the tables' previous readers are done
+    const int chunk_words = kTile * bw / 32;
+    uint32_t *cw = reinterpret_cast<uint32_t *>(ub);
+    {
+        const int64_t cbase = tile * chunk_words;          // the tile's chunk in every code stream
+        const int64_t avail = a.wcode_bytes / 4 - cbase;   // words of the (padded) stream from there
+        const int nvec = n * chunk_words / 4;
+        for (int v = threadIdx.x; v < nvec; v += kThreads) {
+            const int w = (4 * v) / chunk_words, o = (4 * v) % chunk_words;
+            uint4 c = make_uint4(0u, 0u, 0u, 0u);
+            if (o + 4 <= avail)
+                c = __ldg(reinterpret_cast<const uint4 *>(a.wwords + static_cast<int64_t>(w) * a.wwords_stride + cbase + o));
+            reinterpret_cast<uint4 *>(cw)[v] = c;
+        }
+        if (has_scale<QW>())
+            for (int i = threadIdx.x; i < n * ngw; i += kThreads)
+                wsc[i] = __ldg(a.wscales + static_cast<int64_t>(i / ngw) * a.wscales_stride + gw0 + i % ngw);
+        if (seg) cache_tile_groups(GW, tile, d, gs.tg);
+    }
+    compute_sync();
+    float acc[kSlots][4];
+    decode_sum_staged<QW>(a, tile, cw, chunk_words, wsc, ngw, gw0, seg, gs.tg, stab, utab, acc);
+    compute_sync();  // every thread has read the staged codes
+    const float nf = static_cast<float>(n);
+    const bool pow2n = (n & (n - 1)) == 0;
+    const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t q = slot_of(tile, k);
+        const int64_t j0 = 4 * q;
+        float u[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float step = pow2n ? __fmul_rn(acc[k][i], inv_n) : __fdiv_rn(acc[k][i], nf);
+            if (MODE == MODE_S) step = adam_step(step, ms[k][i], vs[k][i], a.hp);
+            u[i] = (in[k] && (FULL || j0 + i < hi)) ? __fadd_rn(step, es[k][i]) : 0.0f;
+        }
+        ub[k * kThreads + threadIdx.x] = make_float4(u[0], u[1], u[2], u[3]);
+        if (MODE == MODE_S && in[k]) {
+            store4<FULL>(a.ms, q, hi, ms[k]);
+            store4<FULL>(a.vs, q, hi, vs[k]);
+        }
+    }
+    return true;
+}
+
+// Algorithm 1 for Q_s scale groups that span tiles, in one cooperative pass (PASS_GROUPED; see
+// GroupPlan and worker_grouped_kernel): phase one decodes, averages and parks w of the CTA's
+// tiles of a wave in shared memory and queues the partial norms, published once per wave; phase
+// two encodes Q_s(w) and stores e_s <- w - Q_s(w).
+template <int MODE, int QW, int QS>
+__global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_grouped_kernel(const ServerArgs a)
+{
+    extern __shared__ __align__(16) float4 uslot[];  // a.gp.slots tiles of w
+    __shared__ GroupSmem gs;
+    __shared__ float utab_s[256];
+    __shared__ float stab[256];
+    __shared__ float wsc[kWorkerScales];
+    build_qtab<QS>(a.qs, gs.qtab);
+    const float *utab = build_worker_utab<QW>(a, utab_s);
+    __syncthreads();
+    const bool staged = server_codes_fit(a, code_bits<QW>(a.qw));
+    const GroupPlan &gp = a.gp;
+    int turn = 0;  // reductions so far (the same count in every thread)
+    for (int w = 0; w < static_cast<int>(gp.n_waves); ++w) {
+        const int64_t c0 = gp.cuts[w], c1 = gp.cuts[w + 1];
+        const int t0 = static_cast<int>(c0 / kTile) + blockIdx.x;   // tiles < 2^28 (d <= 2^40)
+        const int t_end = static_cast<int>((c1 - 1) / kTile) + 1;
+        int k = 0;
+        for (int tile = t0; tile < t_end; tile += gridDim.x, ++k) {
+            float4 *ub = uslot + k * (kThreads * kSlots);
+            const int64_t tl = static_cast<int64_t>(tile) * kTile, lo = max(c0, tl), hi = min(c1, tl + kTile);
+            const bool full = lo == tl && hi == tl + kTile;
+            bool done = false;
+            if (staged)
+                done = full ? server_u_staged<MODE, QW, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs)
+                            : server_u_staged<MODE, QW, false>(a, tile, lo, hi, ub, utab, stab, wsc, gs);
+            if (!done) {
+                compute_sync();  // stab's and tg's previous readers are done
+                if (full) server_u_range<MODE, QW, true>(a, tile, lo, hi, ub, utab, stab, gs.tg);
+                else server_u_range<MODE, QW, false>(a, tile, lo, hi, ub, utab, stab, gs.tg);
+            }
+            range_partials<QS>(ub, tile, lo, hi, a.d, a.qs, a.partials, gs, turn);
+        }
+        if (!wave_barrier(gp, w, a.status, gs)) return;
+        encode_wave<QS>(uslot, t0, t_end, c0, c1, a.d, a.qs, a.words, a.partials, a.scales, a.es, a.ef, a.seed,
+                        static_cast<uint32_t>(a.n), a.t, gs);
+    }
+}
+
+
+constexpr int kWorkerTab = 1024;  // floats of the staged server's per-tile worker table
+
+// Bits 0, 4, ..., 28 of x moved to bits 0 .. 7 (the inverse of spread8_by4).
+__device__ __forceinline__ uint32_t gather_every4(uint32_t x)
+{
+    x &= 0x11111111u;
+    x = (x | (x >> 3)) & 0x03030303u;
+    x = (x | (x >> 6)) & 0x000f000fu;
+    x = (x | (x >> 12)) & 0x000000ffu;
+    return x;
 }
 
 // All 256 compute threads agree on `ok` (named barrier 1 with an AND reduction).
@@ -572,6 +869,40 @@ static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
     }
     server_staged_kernel<MODE, QW, QS><<<a.plan.grid, kThreads + 32, a.plan.smem_bytes, s>>>(a);
     return cudaGetLastError();
+}
+
+
+// The grouped server for one placement and broadcast kind (Q_s with scale groups only).
+template <int MODE, int QS>
+cudaError_t server_grouped_shape_for_qs(int qw, GroupedShape *out)
+{
+    if constexpr (QS != QK_SIGN && QS != QK_UNIF) {
+        return cudaErrorNotSupported;
+    } else {
+        const int w = MODE == MODE_S ? 2 : 3;  // the kernel's launch bounds
+        switch (qw) {
+        case QK_SIGN: return grouped_shape(server_grouped_kernel<MODE, QK_SIGN, QS>, w, out);
+        case QK_UNIF: return grouped_shape(server_grouped_kernel<MODE, QK_UNIF, QS>, w, out);
+        case QK_POW2: return grouped_shape(server_grouped_kernel<MODE, QK_POW2, QS>, w, out);
+        default: return grouped_shape(server_grouped_kernel<MODE, QK_IDENT, QS>, w, out);
+        }
+    }
+}
+
+template <int MODE, int QS>
+cudaError_t launch_server_grouped_for_qs(const ServerArgs &a, int grid, cudaStream_t s)
+{
+    if constexpr (QS != QK_SIGN && QS != QK_UNIF) {
+        return cudaErrorNotSupported;
+    } else {
+        const int slots = a.gp.slots;
+        switch (a.qw.kind) {
+        case QK_SIGN: return grouped_launch(server_grouped_kernel<MODE, QK_SIGN, QS>, a, grid, slots, s);
+        case QK_UNIF: return grouped_launch(server_grouped_kernel<MODE, QK_UNIF, QS>, a, grid, slots, s);
+        case QK_POW2: return grouped_launch(server_grouped_kernel<MODE, QK_POW2, QS>, a, grid, slots, s);
+        default: return grouped_launch(server_grouped_kernel<MODE, QK_IDENT, QS>, a, grid, slots, s);
+        }
+    }
 }
 
 // Launch the server kernel for one placement and one broadcast quantizer kind (each (MODE, QS) pair

@@ -76,10 +76,12 @@ __device__ __forceinline__ bool unif_index_fast(float u, float r, float Lf, floa
 enum EncVar : int { ENC_PLAIN = 0, ENC_UZERO, ENC_UDET_TAB, ENC_UDET_DIV, ENC_USTO_TAB, ENC_USTO_DIV };
 
 // BITS: the code width as a compile-time constant (0: code_bits of the kind, or q.bits).
+// Only the coordinates of [lo, d) are encoded and stored (lo: 0, or the start of a word and a slot).
 template <int QK, bool FULL, bool BALLOT, int VAR, int BITS, class USrc>
 __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t tile, int64_t d,
                                                const QParams &q, uint32_t *words, float *resid, int ef,
-                                               uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
+                                               uint64_t seed, uint32_t id, uint32_t t, const float *qtab,
+                                               int64_t lo = 0)
 {
     constexpr bool STO = VAR == ENC_USTO_TAB || VAR == ENC_USTO_DIV;
     constexpr bool TAB = VAR == ENC_UDET_TAB || VAR == ENC_USTO_TAB;
@@ -87,7 +89,6 @@ __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t
     const int bits = BITS ? BITS : code_bits<QK>(q);
     const int L = (QK == QK_UNIF) ? unif_L(bits) : 0;
     const float Lf = static_cast<float>(L);
-    const int64_t n_words = (d * bits + 31) >> 5;
     float r = 0.0f, m = 0.0f;
     if (GRID) {
         r = (s >= 0x1p-125f && s <= 0x1p125f) ? __frcp_rn(s) : __int_as_float(0x7fc00000);
@@ -130,8 +131,8 @@ __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t
             c[i] = (FULL || j0 + i < d) ? code : 0u;
             e[i] = ef ? __fsub_rn(uk[i], dec) : 0.0f;
         }
-        store_codes4<FULL, BALLOT>(words, qs, bits, c, n_words);
-        if (ef && (FULL || j0 < d)) store4<FULL>(resid, qs, d, e);
+        store_codes4<FULL, BALLOT>(words, qs, bits, c, lo, d);
+        if (ef && (FULL || (j0 >= lo && j0 < d))) store4<FULL>(resid, qs, d, e);
     }
 }
 
@@ -142,39 +143,41 @@ __device__ __forceinline__ void encode_store_v(const USrc &src, float s, int64_t
 template <int QK, bool FULL, bool BALLOT, int BITS, class USrc>
 __device__ __forceinline__ void encode_store_unif(const USrc &u, float s, int64_t tile, int64_t d,
                                                   const QParams &q, uint32_t *words, float *resid, int ef,
-                                                  uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
+                                                  uint64_t seed, uint32_t id, uint32_t t, const float *qtab,
+                                                  int64_t lo = 0)
 {
     constexpr bool tab = BITS <= 8;
     if (!(s > 0.0f))
-        encode_store_v<QK, FULL, BALLOT, ENC_UZERO, BITS>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        encode_store_v<QK, FULL, BALLOT, ENC_UZERO, BITS>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo);
     else if (q.stochastic)
         encode_store_v<QK, FULL, BALLOT, tab ? ENC_USTO_TAB : ENC_USTO_DIV, BITS>(u, s, tile, d, q, words, resid, ef,
-                                                                               seed, id, t, qtab);
+                                                                               seed, id, t, qtab, lo);
     else
         encode_store_v<QK, FULL, BALLOT, tab ? ENC_UDET_TAB : ENC_UDET_DIV, BITS>(u, s, tile, d, q, words, resid, ef,
-                                                                               seed, id, t, qtab);
+                                                                               seed, id, t, qtab, lo);
 }
 
 // Encode and store a tile; the variant (and a configured code width) is chosen once per tile.
 template <int QK, bool FULL, bool BALLOT, class USrc>
 __device__ __forceinline__ void encode_store(const USrc &u, float s, int64_t tile, int64_t d,
                                              const QParams &q, uint32_t *words, float *resid, int ef,
-                                             uint64_t seed, uint32_t id, uint32_t t, const float *qtab)
+                                             uint64_t seed, uint32_t id, uint32_t t, const float *qtab,
+                                             int64_t lo = 0)
 {
     if constexpr (QK == QK_UNIF) {
         switch (q.bits) {  // the widths ea_init accepts
-        case 2: encode_store_unif<QK, FULL, BALLOT, 2>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
-        case 4: encode_store_unif<QK, FULL, BALLOT, 4>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
-        case 8: encode_store_unif<QK, FULL, BALLOT, 8>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
-        default: encode_store_unif<QK, FULL, BALLOT, 16>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab); break;
+        case 2: encode_store_unif<QK, FULL, BALLOT, 2>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo); break;
+        case 4: encode_store_unif<QK, FULL, BALLOT, 4>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo); break;
+        case 8: encode_store_unif<QK, FULL, BALLOT, 8>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo); break;
+        default: encode_store_unif<QK, FULL, BALLOT, 16>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo); break;
         }
     } else if constexpr (QK == QK_POW2) {
         if (q.bits == 4)
-            encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 4>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+            encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 4>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo);
         else
-            encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 8>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+            encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 8>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo);
     } else {
-        encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 0>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab);
+        encode_store_v<QK, FULL, BALLOT, ENC_PLAIN, 0>(u, s, tile, d, q, words, resid, ef, seed, id, t, qtab, lo);
     }
 }
 

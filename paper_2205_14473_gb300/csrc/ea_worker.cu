@@ -1,5 +1,5 @@
 // ea_worker.cu -- worker compress (Algorithm 2), the two-pass scale kernels, and x <- x - Q_s(w).
-#include "ea_tile.cuh"
+#include "ea_grouped.cuh"
 
 namespace ea {
 
@@ -71,6 +71,85 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 3)
     }
 }
 
+// Phase one of a grouped worker tile: u of the coordinate range [lo, hi) of tile `tile` (0
+// elsewhere) into ub, with m and v updated and stored in the range (Adam at the worker).
+// FULL: the range is the whole tile.  All four slots' loads are issued at once (the kernel's
+// register budget is sized for it), so that enough bytes are in flight per SM.
+template <int MODE, bool FULL>
+__device__ __forceinline__ void worker_u_range(const WorkerArgs &a, int64_t tile, int64_t lo, int64_t hi, float4 *ub)
+{
+    constexpr int H = kSlots;
+#pragma unroll
+    for (int h = 0; h < kSlots; h += H) {
+        float g[H][4], e[H][4], m[H][4], v[H][4];
+        bool in[H];
+#pragma unroll
+        for (int k = 0; k < H; ++k) {
+            const int64_t q = slot_of(tile, h + k);
+            in[k] = FULL || (4 * q >= lo && 4 * q < hi);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) g[k][i] = e[k][i] = m[k][i] = 0.0f, v[k][i] = 1.0f;
+            if (in[k]) {
+                load4<FULL>(a.g, q, hi, g[k]);
+                load4<FULL>(a.e, q, hi, e[k]);
+                if (MODE == MODE_W) {
+                    load4<FULL>(a.m, q, hi, m[k]);
+                    load4<FULL>(a.v, q, hi, v[k]);
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < H; ++k) {
+            const int64_t q = slot_of(tile, h + k);
+            const int64_t j0 = 4 * q;
+            float u[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                float step = g[k][i];
+                if (MODE == MODE_W) step = adam_step(g[k][i], m[k][i], v[k][i], a.hp);
+                u[i] = (in[k] && (FULL || j0 + i < hi)) ? __fadd_rn(step, e[k][i]) : 0.0f;
+            }
+            ub[(h + k) * kThreads + threadIdx.x] = make_float4(u[0], u[1], u[2], u[3]);
+            if (MODE == MODE_W && in[k]) {
+                store4<FULL>(a.m, q, hi, m[k]);
+                store4<FULL>(a.v, q, hi, v[k]);
+            }
+        }
+    }
+}
+
+// Algorithm 2 for scale groups that span tiles, in one cooperative pass (PASS_GROUPED; see
+// GroupPlan): for each wave, every CTA computes u of its tiles into shared memory (phase one) and
+// publishes the partial norms; once a group's scale is ready, the tiles are encoded from shared
+// memory and e <- u - Q_w(u) stored (phase two).  HBM traffic per coordinate as worker_kernel's:
+// no second read of u.
+template <int MODE, int QK>
+__global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 2) worker_grouped_kernel(const WorkerArgs a)
+{
+    extern __shared__ __align__(16) float4 uslot[];  // a.gp.slots tiles of u
+    __shared__ GroupSmem gs;
+    build_qtab<QK>(a.q, gs.qtab);
+    __syncthreads();
+    const GroupPlan &gp = a.gp;
+    int turn = 0;  // reductions so far (the same count in every thread)
+    for (int w = 0; w < static_cast<int>(gp.n_waves); ++w) {
+        const int64_t c0 = gp.cuts[w], c1 = gp.cuts[w + 1];
+        const int t0 = static_cast<int>(c0 / kTile) + blockIdx.x;   // tiles < 2^28 (d <= 2^40)
+        const int t_end = static_cast<int>((c1 - 1) / kTile) + 1;
+        int k = 0;
+        for (int tile = t0; tile < t_end; tile += gridDim.x, ++k) {
+            float4 *ub = uslot + k * (kThreads * kSlots);
+            const int64_t tl = static_cast<int64_t>(tile) * kTile, lo = max(c0, tl), hi = min(c1, tl + kTile);
+            if (lo == tl && hi == tl + kTile) worker_u_range<MODE, true>(a, tile, lo, hi, ub);
+            else worker_u_range<MODE, false>(a, tile, lo, hi, ub);
+            range_partials<QK>(ub, tile, lo, hi, a.d, a.q, a.partials, gs, turn);
+        }
+        if (!wave_barrier(gp, w, a.status, gs)) return;
+        encode_wave<QK>(uslot, t0, t_end, c0, c1, a.d, a.q, a.words, a.partials, a.scales, a.e, a.ef, a.seed, a.id,
+                        a.t, gs);
+    }
+}
+
 // Second pass, one CTA per scale group: combine the group's per-tile partial norms in a fixed
 // order and write the group scale (Example 1: ||.||_inf; scaled sign: ||.||_1 / |group|).
 template <int QK>
@@ -110,7 +189,6 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
     const Grouping &G = a.q.grp;
     const int L = (QK == QK_UNIF) ? unif_L(a.q.bits) : 0;
     const float Lf = static_cast<float>(L);
-    const int64_t n_words = (d * a.q.bits + 31) >> 5;
     const int64_t hint = first_group_of_tile(G, tile);
     float u[kSlots][4];
 #pragma unroll
@@ -149,7 +227,7 @@ __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
             }
             e[i] = a.ef ? __fsub_rn(u[k][i], dec) : 0.0f;
         }
-        store_codes4(a.words, qs, a.q.bits, c, n_words);
+        store_codes4(a.words, qs, a.q.bits, c, 0, d);
         if (j0 < d) store4(a.buf, qs, d, e);
     }
 }
@@ -282,6 +360,27 @@ static cudaError_t launch_worker_mode(const WorkerArgs &a, cudaStream_t s)
 cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s)
 {
     return mode == MODE_W ? launch_worker_mode<MODE_W>(a, s) : launch_worker_mode<MODE_S>(a, s);
+}
+
+// The grouped kernels exist for the quantizers with scale groups (scaled sign, uniform grid).
+cudaError_t worker_grouped_shape(int mode, int qk, GroupedShape *out)
+{
+    const int w = mode == MODE_W ? 2 : 4;  // the kernels' launch bounds
+    if (mode == MODE_W && qk == QK_SIGN) return grouped_shape(worker_grouped_kernel<MODE_W, QK_SIGN>, w, out);
+    if (mode == MODE_W && qk == QK_UNIF) return grouped_shape(worker_grouped_kernel<MODE_W, QK_UNIF>, w, out);
+    if (mode == MODE_S && qk == QK_SIGN) return grouped_shape(worker_grouped_kernel<MODE_S, QK_SIGN>, w, out);
+    if (mode == MODE_S && qk == QK_UNIF) return grouped_shape(worker_grouped_kernel<MODE_S, QK_UNIF>, w, out);
+    return cudaErrorNotSupported;
+}
+
+cudaError_t launch_worker_grouped(int mode, const WorkerArgs &a, int grid, cudaStream_t s)
+{
+    const int slots = a.gp.slots;
+    if (mode == MODE_W && a.q.kind == QK_SIGN) return grouped_launch(worker_grouped_kernel<MODE_W, QK_SIGN>, a, grid, slots, s);
+    if (mode == MODE_W && a.q.kind == QK_UNIF) return grouped_launch(worker_grouped_kernel<MODE_W, QK_UNIF>, a, grid, slots, s);
+    if (mode == MODE_S && a.q.kind == QK_SIGN) return grouped_launch(worker_grouped_kernel<MODE_S, QK_SIGN>, a, grid, slots, s);
+    if (mode == MODE_S && a.q.kind == QK_UNIF) return grouped_launch(worker_grouped_kernel<MODE_S, QK_UNIF>, a, grid, slots, s);
+    return cudaErrorNotSupported;
 }
 
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s)

@@ -131,6 +131,40 @@ def test_staged_server_several_tiles_per_cta(qw, qs, placement):
     _run_host(cfg, 2, seed=37, grad_scale=1e-3)
 
 
+def test_two_pass_scale_beyond_the_grouped_capacity():
+    """A whole-vector scale over 12.3 million coordinates: more tiles than the one-pass grouped
+    kernels hold in shared memory at once (about 1,800 on a GB300), so both messages take the
+    two-pass scale (stash, finalize, encode: three launches each)."""
+    d = 3000 * 4096 + 3
+    cfg = ea.EAConfig(d=d, n=2, qw=W.sign_q(0), qs=W.uniform_q(8, 0, False), alpha=1e-3, seed=41)
+    L = _run_host(cfg, 2, seed=43)
+    assert L.gpu.launches_per_round == 2 * 3 + 3 + 1
+
+
+@pytest.mark.parametrize("qw,qs", [(W.sign_q(0), W.sign_q(0)), (W.uniform_q(4, 0, True), W.uniform_q(8, 1000, False))])
+def test_grouped_scales_one_launch_per_message(qw, qs):
+    """Scale groups that span tiles take the one-pass grouped kernels (74 tiles: one per worker CTA):
+    one launch per message."""
+    cfg = ea.EAConfig(d=300_001, n=3, qw=qw, qs=qs, alpha=1e-3, seed=45)
+    L = _run_host(cfg, 3, seed=47)
+    assert L.gpu.launches_per_round == 3 + 1 + 1
+
+
+@pytest.mark.parametrize("qw,qs,placement", [
+    (W.sign_q(0), W.sign_q(0), ea.ADAM_AT_WORKER),
+    (W.uniform_q(4, 0, True), W.uniform_q(8, 0, False), ea.ADAM_AT_SERVER),
+    (W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)), W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)),
+     ea.ADAM_AT_WORKER),
+])
+def test_grouped_broadcast_with_several_tiles_per_cta(qw, qs, placement):
+    """4.4 million coordinates (1,075 tiles): the grouped broadcast's CTAs each hold several tiles
+    of one wave, while the workers' messages take the two-pass scale."""
+    d = 4_400_200
+    cfg = ea.EAConfig(d=d, n=3, qw=qw, qs=qs, alpha=1e-3, placement=placement, seed=49)
+    L = _run_host(cfg, 2, seed=51)
+    assert L.gpu.launches_per_round == 3 * 3 + 1 + 1
+
+
 def test_replicas_are_identical_and_protocol():
     cfg = ea.EAConfig(d=10_000, n=2, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-3)
     rnd = ea.EARound(cfg)
@@ -181,6 +215,7 @@ def test_c1_full():
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
     assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (2_622_720, 2_622_720)
+    assert L.gpu.launches_per_round == w.n + 2  # whole-vector scales in one pass per message
 
 
 def test_c2_quadratic_toy_full():
@@ -221,6 +256,8 @@ def test_c3_resnet18_all_tensors(placement, rounds):
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
     assert L.total_mismatch == 0
+    # per-tensor scales: the broadcast in one grouped pass; the 2,854-tile worker messages in two
+    assert L.gpu.launches_per_round == 3 * w.n + 2
     if rounds == w.rounds:
         assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (18_706_393_600, 18_706_393_600)
 
