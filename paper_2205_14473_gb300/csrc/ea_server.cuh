@@ -508,10 +508,12 @@ __device__ __forceinline__ void transpose8x8(uint32_t &lo, uint32_t &hi)
 // cache; the slots and coordinates inside it are unrolled.
 // PAIRS (B = 4): the thread-pair decode below (used with Adam at the workers; with Adam at the
 // server the per-thread form measured faster, the Adam step leaving fewer registers).
-template <int B, bool PAIRS>
-__device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int n, const float *wtab,
+// NW > 0: the worker count n is NW, known at compile time (the worker loop is then unrolled).
+template <int B, bool PAIRS, int NW = 0>
+__device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int n_rt, const float *wtab,
                                                 float (&acc)[kSlots][4])
 {
+    const int n = NW ? NW : n_rt;
     constexpr int chunk_words = kTile * B / 32;
     constexpr uint32_t mask = (1u << B) - 1u;
     // the slot's 4B bits start at bit 4 B ls of the chunk, ls = k * kThreads + threadIdx.x
@@ -530,7 +532,7 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
         for (int h = 0; h < kSlots / 2; ++h)
 #pragma unroll
             for (int j = 0; j < 8; ++j) blk[h][j] = 0.0f;
-#pragma unroll 2
+#pragma unroll(NW ? NW : 2)
         for (int w = 0; w < n; ++w, pw += chunk_words, tb += 4 << B) {
 #pragma unroll
             for (int h = 0; h < kSlots / 2; ++h) {
@@ -557,7 +559,7 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
     const int sh = ((static_cast<int>(threadIdx.x) * B) & 7) * 4;
     const uint32_t *cw = reinterpret_cast<const uint32_t *>(codes) + ((static_cast<int>(threadIdx.x) * B) >> 3);
     const unsigned char *tb = reinterpret_cast<const unsigned char *>(wtab);
-#pragma unroll 2
+#pragma unroll(NW ? NW : 2)
     for (int w = 0; w < n; ++w, cw += chunk_words, tb += 4 << B) {
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
@@ -576,19 +578,22 @@ __device__ __forceinline__ void unif_decode_sum(const unsigned char *codes, int 
 // One tile of the staged server on the compute warps: the stage `st` holds e_s (m_s, v_s), the
 // workers' code chunks and scales.  The stage's e_s slots then hold u until the re-quantization
 // has read it; the stage is released (arrive on `empty`) after that.
-// SMALLN: n <= 8 is known at compile time (the scaled-sign table then is the whole average and the
-// per-worker path is not compiled in for scaled-sign workers).
-template <int MODE, int QW, int QS, bool FULL, bool SMALLN>
+// NW: the worker count when it is 8, known at compile time (the per-worker bounds, the average's
+// division and the decode loops then fold; for scaled-sign workers the table is the whole average
+// and the per-worker path is not compiled in), or 0 for a count known at run time.
+template <int MODE, int QW, int QS, bool FULL, int NW>
 __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t tile, const unsigned char *st,
                                                    bool ok, uint64_t *empty, int Lw, float Lwf, const float *utab,
                                                    float *wtab, const uint32_t (&flip)[8], TileSmem &sm)
 {
+    static_assert(NW == 0 || NW == 8, "a compile-time worker count of 8");
     const StagePlan &P = a.plan;
     const int64_t d = a.d;
     const int bw = code_bits<QW>(a.qw);
-    const float nf = static_cast<float>(a.n);
-    const bool pow2n = (a.n & (a.n - 1)) == 0;
-    const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
+    const int n = NW ? NW : a.n;
+    const float nf = static_cast<float>(n);
+    const bool pow2n = (n & (n - 1)) == 0;
+    const float inv_n = NW ? 1.0f / NW : __frcp_rn(nf);  // exact when n is a power of two
     float acc[kSlots][4];  // the average of the decoded worker messages
     const float *sc = reinterpret_cast<const float *>(st + P.off_scales);
     bool done = false;
@@ -597,7 +602,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
     if constexpr (!has_scale<QS>() && (QW == QK_SIGN || QW == QK_UNIF)) compute_sync();
     if constexpr (QW == QK_SIGN) {
       {
-        done = SMALLN || a.n <= 8;
+        done = NW == 8 || n <= 8;
         // Scaled-sign workers: the worker-order sum of the first m = min(n, 8) workers depends
         // only on their m sign bits.  Thread p forms it for sign pattern p (bit w = worker w's
         // code), exactly as the per-coordinate loop would; for n <= 8 it is divided by n and is
@@ -606,7 +611,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
             float t = 0.0f;
 #pragma unroll
             for (int w = 0; w < 8; ++w)
-                if (w < a.n) t = __fadd_rn(t, __uint_as_float(__float_as_uint(sc[w]) ^ flip[w]));
+                if (w < n) t = __fadd_rn(t, __uint_as_float(__float_as_uint(sc[w]) ^ flip[w]));
             wtab[threadIdx.x] = !done ? t : pow2n ? __fmul_rn(t, inv_n) : __fdiv_rn(t, nf);
         }
         // the table's barrier, and agreement on the stage wait: if any thread's wait ran out, the
@@ -628,7 +633,7 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
             const int word = 32 * (k + (odd ? 1 : 0)) + static_cast<int>(threadIdx.x >> 3);
             uint32_t wd[8];
 #pragma unroll
-            for (int w = 0; w < 8; ++w) wd[w] = w < a.n ? c0[w * (kTile / 32) + word] : 0u;
+            for (int w = 0; w < 8; ++w) wd[w] = w < n ? c0[w * (kTile / 32) + word] : 0u;
             uint32_t lo = __byte_perm(__byte_perm(wd[0], wd[1], sel), __byte_perm(wd[2], wd[3], sel), 0x5410);
             uint32_t hi = __byte_perm(__byte_perm(wd[4], wd[5], sel), __byte_perm(wd[6], wd[7], sel), 0x5410);
             transpose8x8(lo, hi);
@@ -658,9 +663,9 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
         // decode1 would form them, so that a coordinate's decode is one table read.
         // Worker w's table starts at w * 2^b; entries 0 .. 2L = 2^b - 2 are used.
         const int nL = 2 * Lw + 1;
-        const bool dec_tab = QW == QK_UNIF && utab != nullptr && (a.n << bw) <= kWorkerTab;
+        const bool dec_tab = QW == QK_UNIF && utab != nullptr && (n << bw) <= kWorkerTab;
         if (dec_tab) {
-            for (int idx = threadIdx.x; idx < (a.n << bw); idx += kThreads) {
+            for (int idx = threadIdx.x; idx < (n << bw); idx += kThreads) {
                 const int i = idx & ((1 << bw) - 1);
                 if (i < nL) wtab[idx] = __fmul_rn(sc[idx >> bw], utab[i]);
             }
@@ -670,16 +675,16 @@ __device__ __forceinline__ bool server_staged_tile(const ServerArgs &a, int64_t 
         bool summed = false;
         if constexpr (QW == QK_UNIF) {
             if (dec_tab && bw == 4) {
-                unif_decode_sum<4, MODE == MODE_W>(st + P.off_codes, a.n, wtab, acc);
+                unif_decode_sum<4, MODE == MODE_W, NW>(st + P.off_codes, n, wtab, acc);
                 summed = true;
             } else if (dec_tab && bw == 8) {
-                unif_decode_sum<8, false>(st + P.off_codes, a.n, wtab, acc);
+                unif_decode_sum<8, false, NW>(st + P.off_codes, n, wtab, acc);
                 summed = true;
             }
         }
         if (!summed) {  // any worker count and code width; kept rolled (it is not the common case)
 #pragma unroll 1
-            for (int w = partial ? 8 : 0; w < a.n; ++w) {
+            for (int w = partial ? 8 : 0; w < n; ++w) {
                 const uint32_t *cw = reinterpret_cast<const uint32_t *>(st + P.off_codes + static_cast<size_t>(w) * P.code_chunk);
                 const float sw = has_scale<QW>() ? sc[w] : 0.0f;
                 const float *dw = wtab + (w << bw);
@@ -830,7 +835,7 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
     uint32_t flip[8];
 #pragma unroll
     for (int w = 0; w < 8; ++w) flip[w] = ((threadIdx.x >> w) & 1u) ? 0u : 0x80000000u;
-    const bool small = QW == QK_SIGN && a.n <= 8;  // full tiles of scaled-sign workers: SMALLN
+    const bool n8 = a.n == 8;  // full tiles with eight workers: the compile-time count
     int64_t it = 0;
     for (int64_t tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++it) {
         const int s = static_cast<int>(it % S);
@@ -838,9 +843,9 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
         const bool ok = mbar_wait(&full[s], static_cast<uint32_t>((it / S) & 1));
         const unsigned char *st = stage0 + static_cast<size_t>(s) * P.stage_bytes;
         const bool go = (tile + 1) * kTile <= d
-            ? (small ? server_staged_tile<MODE, QW, QS, true, true>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm)
-                     : server_staged_tile<MODE, QW, QS, true, false>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm))
-            : server_staged_tile<MODE, QW, QS, false, false>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
+            ? (n8 ? server_staged_tile<MODE, QW, QS, true, 8>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm)
+                  : server_staged_tile<MODE, QW, QS, true, 0>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm))
+            : server_staged_tile<MODE, QW, QS, false, 0>(a, tile, st, ok, &empty[s], Lw, Lwf, use_tab ? utab : nullptr, wtab, flip, sm);
         if (!go) {
             if (threadIdx.x == 0) report_status(a.status, kStatusTimeout);
             break;
