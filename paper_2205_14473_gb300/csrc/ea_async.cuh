@@ -7,6 +7,8 @@
 #pragma once
 
 #include <cstdint>
+#include <utility>
+
 #include <cuda_runtime.h>
 
 namespace ea {
@@ -92,6 +94,33 @@ __device__ __forceinline__ void cp_async_arrive_noinc(uint64_t *bar)
 __device__ __forceinline__ void report_status(uint32_t *status, uint32_t code)
 {
     if (status) atomicOr(status, code);
+}
+
+// Programmatic dependent launch.  The round's kernels are launched with programmatic stream
+// serialization (launch_pdl): each lets the next kernel on the stream be scheduled as soon as all of
+// its own CTAs have started (pdl_trigger), and each waits, before its first access to global
+// memory, until the previous kernel has completed and its writes are visible (pdl_wait).  The next
+// kernel's launch and shared-memory prologue thus overlap this one's last CTAs; the data order of
+// the stream is unchanged.  Without the launch attribute both are no-ops.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Launch `kernel` with programmatic stream serialization (see pdl_trigger / pdl_wait).
+template <class... KArgs, class... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args &&...args)
+{
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 }  // namespace ea

@@ -141,9 +141,11 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
     const int64_t tile = blockIdx.x;
     const int64_t d = a.d;
 
+    pdl_trigger();
     build_qtab<QS>(a.qs, sm.qtab);  // read after the scale reduction's barrier
     const float *utab = build_worker_utab<QW>(a, utab_s);
     if (utab) __syncthreads();
+    pdl_wait();
 
     float es[kSlots][4], ms[kSlots][4], vs[kSlots][4];
 #pragma unroll
@@ -773,6 +775,7 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
     unsigned char *stage0 = dsm + 128 * ((2 * S * 8 + 127) / 128);
     constexpr bool scaled_w = has_scale<QW>();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    pdl_trigger();
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -788,6 +791,7 @@ __global__ void __launch_bounds__(kThreads + 32, server_ctas_per_sm(MODE, QW, QS
         for (int i = threadIdx.x; i <= 2 * Lw; i += blockDim.x) utab[i] = __fdiv_rn(static_cast<float>(i - Lw), Lwf);
     build_qtab<QS>(a.qs, sm.qtab);
     __syncthreads();
+    pdl_wait();  // the workers' messages and e_s are written
 
     if (warp == kWarps) {  // ---------------------------------------------------------- producer
         int64_t it = 0;
@@ -872,8 +876,7 @@ static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
         if (e != cudaSuccess) return e;
         attr_set[dev].store(true, std::memory_order_release);
     }
-    server_staged_kernel<MODE, QW, QS><<<a.plan.grid, kThreads + 32, a.plan.smem_bytes, s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(server_staged_kernel<MODE, QW, QS>, dim3(a.plan.grid), dim3(kThreads + 32), a.plan.smem_bytes, s, a);
 }
 
 
@@ -919,20 +922,16 @@ cudaError_t launch_server_for_qs(const ServerArgs &a, cudaStream_t s)
     switch (a.qw.kind) {
     case QK_SIGN:
         if (a.plan.enabled) return launch_server_staged<MODE, QK_SIGN, QS>(a, s);
-        server_kernel<MODE, QK_SIGN, QS><<<grid, block, 0, s>>>(a);
-        break;
+        return launch_pdl(server_kernel<MODE, QK_SIGN, QS>, grid, block, 0, s, a);
     case QK_UNIF:
         if (a.plan.enabled) return launch_server_staged<MODE, QK_UNIF, QS>(a, s);
-        server_kernel<MODE, QK_UNIF, QS><<<grid, block, 0, s>>>(a);
-        break;
+        return launch_pdl(server_kernel<MODE, QK_UNIF, QS>, grid, block, 0, s, a);
     case QK_POW2:
         if (a.plan.enabled) return launch_server_staged<MODE, QK_POW2, QS>(a, s);
-        server_kernel<MODE, QK_POW2, QS><<<grid, block, 0, s>>>(a);
-        break;
+        return launch_pdl(server_kernel<MODE, QK_POW2, QS>, grid, block, 0, s, a);
     default:
         if (a.plan.enabled) return launch_server_staged<MODE, QK_IDENT, QS>(a, s);
-        server_kernel<MODE, QK_IDENT, QS><<<grid, block, 0, s>>>(a);
-        break;
+        return launch_pdl(server_kernel<MODE, QK_IDENT, QS>, grid, block, 0, s, a);
     }
     return cudaGetLastError();
 }

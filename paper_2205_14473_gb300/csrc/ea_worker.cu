@@ -59,6 +59,8 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 3)
 {
     __shared__ TileSmem sm;
     __shared__ float4 ubuf[kSlots * kThreads];
+    pdl_trigger();
+    pdl_wait();
     const int64_t tile = blockIdx.x;
     // the scale pass as a compile-time constant: each instantiation carries only its own path
     const bool full = (tile + 1) * kTile <= a.d;
@@ -156,6 +158,8 @@ template <int QK>
 __global__ void __launch_bounds__(kThreads) finalize_kernel(const FinalizeArgs a)
 {
     __shared__ double red[kWarps];
+    pdl_trigger();
+    pdl_wait();
     const int64_t gi = blockIdx.x;
     const int64_t pb = a.q.grp.pair_base[gi], pe = a.q.grp.pair_base[gi + 1];
     double acc = 0.0;
@@ -182,8 +186,10 @@ template <int QK>
 __global__ void __launch_bounds__(kThreads, 2) encode_kernel(const EncodeArgs a)
 {
     __shared__ float qtab_s[256];
+    pdl_trigger();
     const float *qtab = build_qtab<QK>(a.q, qtab_s);
     __syncthreads();
+    pdl_wait();
     const int64_t tile = blockIdx.x;
     const int64_t d = a.d;
     const Grouping &G = a.q.grp;
@@ -320,6 +326,8 @@ template <int QK>
 __global__ void __launch_bounds__(kThreads) apply_kernel(const ApplyArgs a)
 {
     __shared__ float qtab_s[256];
+    pdl_trigger();
+    pdl_wait();
     if constexpr (QK == QK_UNIF) {
         switch (a.q.bits) {  // the widths ea_init accepts
         case 2: apply_body<QK, 2>(a, qtab_s); break;
@@ -349,12 +357,11 @@ static cudaError_t launch_worker_mode(const WorkerArgs &a, cudaStream_t s)
 {
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
     switch (a.q.kind) {
-    case QK_SIGN: worker_kernel<MODE, QK_SIGN><<<grid, block, 0, s>>>(a); break;
-    case QK_UNIF: worker_kernel<MODE, QK_UNIF><<<grid, block, 0, s>>>(a); break;
-    case QK_POW2: worker_kernel<MODE, QK_POW2><<<grid, block, 0, s>>>(a); break;
-    default: worker_kernel<MODE, QK_IDENT><<<grid, block, 0, s>>>(a); break;
+    case QK_SIGN: return launch_pdl(worker_kernel<MODE, QK_SIGN>, grid, block, 0, s, a);
+    case QK_UNIF: return launch_pdl(worker_kernel<MODE, QK_UNIF>, grid, block, 0, s, a);
+    case QK_POW2: return launch_pdl(worker_kernel<MODE, QK_POW2>, grid, block, 0, s, a);
+    default: return launch_pdl(worker_kernel<MODE, QK_IDENT>, grid, block, 0, s, a);
     }
-    return cudaGetLastError();
 }
 
 cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s)
@@ -386,29 +393,26 @@ cudaError_t launch_worker_grouped(int mode, const WorkerArgs &a, int grid, cudaS
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s)
 {
     const dim3 grid(static_cast<unsigned>(a.q.grp.n_groups)), block(kThreads);
-    if (a.q.kind == QK_SIGN) finalize_kernel<QK_SIGN><<<grid, block, 0, s>>>(a);
-    else finalize_kernel<QK_UNIF><<<grid, block, 0, s>>>(a);
-    return cudaGetLastError();
+    if (a.q.kind == QK_SIGN) return launch_pdl(finalize_kernel<QK_SIGN>, grid, block, 0, s, a);
+    return launch_pdl(finalize_kernel<QK_UNIF>, grid, block, 0, s, a);
 }
 
 cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s)
 {
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
-    if (a.q.kind == QK_SIGN) encode_kernel<QK_SIGN><<<grid, block, 0, s>>>(a);
-    else encode_kernel<QK_UNIF><<<grid, block, 0, s>>>(a);
-    return cudaGetLastError();
+    if (a.q.kind == QK_SIGN) return launch_pdl(encode_kernel<QK_SIGN>, grid, block, 0, s, a);
+    return launch_pdl(encode_kernel<QK_UNIF>, grid, block, 0, s, a);
 }
 
 cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s)
 {
     const dim3 grid(static_cast<unsigned>((a.d + kTile - 1) / kTile)), block(kThreads);
     switch (a.q.kind) {
-    case QK_SIGN: apply_kernel<QK_SIGN><<<grid, block, 0, s>>>(a); break;
-    case QK_UNIF: apply_kernel<QK_UNIF><<<grid, block, 0, s>>>(a); break;
-    case QK_POW2: apply_kernel<QK_POW2><<<grid, block, 0, s>>>(a); break;
-    default: apply_kernel<QK_IDENT><<<grid, block, 0, s>>>(a); break;
+    case QK_SIGN: return launch_pdl(apply_kernel<QK_SIGN>, grid, block, 0, s, a);
+    case QK_UNIF: return launch_pdl(apply_kernel<QK_UNIF>, grid, block, 0, s, a);
+    case QK_POW2: return launch_pdl(apply_kernel<QK_POW2>, grid, block, 0, s, a);
+    default: return launch_pdl(apply_kernel<QK_IDENT>, grid, block, 0, s, a);
     }
-    return cudaGetLastError();
 }
 
 cudaError_t launch_fill(float *p, int64_t count, float value, cudaStream_t s)
