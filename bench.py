@@ -115,6 +115,20 @@ def _ncu_traffic(kernel: str, workload: str, placement: int):
     return None
 
 
+# The kernels behind each step of a round (a message of the two-pass scale is three launches).
+ROLE_KERNELS = {"compress": ("worker_kernel", "worker_grouped", "finalize_kernel", "encode_kernel"),
+                "server": ("server_staged", "server_grouped", "server_kernel"),
+                "apply": ("apply_kernel",)}
+
+
+def _ncu_traffic_role(role: str, workload: str, placement: int):
+    """Summed per-launch DRAM bytes of the kernels that make up one step of a round, from the
+    committed ncu summary, if every such row was taken on the current kernel sources."""
+    vals = [_ncu_traffic(k, workload, placement) for k in ROLE_KERNELS[role]]
+    vals = [v for v in vals if v is not None]
+    return sum(vals) if vals else None
+
+
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
 
@@ -350,7 +364,8 @@ class RoundTimer:
             ms = statistics.mean(ts)
             gbs = ab[name] / (ms / 1e3) / 1e9
             out[name] = {"ms": ms, "min_ms": min(ts), "gbs": gbs, "frac_measured": gbs / peak,
-                         "frac_8tbs": gbs / NOMINAL_HBM_GBS, "bytes": ab[name]}
+                         "frac_8tbs": gbs / NOMINAL_HBM_GBS, "bytes": ab[name],
+                         "traffic": _ncu_traffic_role(name, self.w.name, self.placement)}
         rgbs = ab["round"] / (ms_total / steps / 1e3) / 1e9
         out["round"] = {"gbs": rgbs, "frac_measured": rgbs / peak, "frac_8tbs": rgbs / NOMINAL_HBM_GBS,
                         "bytes": ab["round"]}
