@@ -128,16 +128,27 @@ int ea_bits_sent(const ea_handle *h, uint64_t *up_bits, uint64_t *down_bits);
 int ea_round_index(const ea_handle *h, int64_t *t);
 
 /* Kernel launches that one round makes on the stream: n worker compresses, one server step and one
- * apply.  A message takes one launch, or three when its scale groups span 4096-coordinate tiles
- * and the one-pass grouped kernel is not used for it: the two-pass scale then adds a finalize and
- * an encode.  The broadcast takes the grouped kernel whenever its waves fit the device's shared
- * memory (groups of up to ~7.5 million coordinates on a GB300); the workers' messages only when
- * the vector has no more 4096-tiles than the grouped kernel has resident CTAs. */
+ * apply.  A message whose scale groups lie inside 4096-coordinate tiles takes one launch.  When the
+ * groups span tiles:
+ *   - a scaled-sign message takes two: one pass writes the codes (the signs, which need no scale)
+ *     with the groups' partial norms, and a finalize forms the scales (the residual is formed from
+ *     the kept input where it is next read; see the residual views);
+ *   - another message takes one launch in the grouped kernel, which holds u in shared memory while
+ *     the partial norms are combined, when its waves fit: for the broadcast, groups of up to ~7.5
+ *     million coordinates on a GB300; for a worker message, no more 4096-tiles than the grouped
+ *     kernel has resident CTAs;
+ *   - otherwise three: the two-pass scale (stash, finalize, encode). */
 int ea_round_launches(const ea_handle *h, int32_t *launches);
 
 /* Device views into the workspace (for inspection and checkpoints); index = worker for per-worker
  * views, ignored otherwise.  *bytes receives the view's size.  A view that does not exist in the
- * configured placement returns EA_E_INVAL. */
+ * configured placement returns EA_E_INVAL.
+ * A scaled-sign message whose groups span tiles keeps its quantizer's input (u of a worker, w of
+ * the server) in place of the residual, which is formed from that input and the message's scales,
+ * e = u - Q(u), where it is next needed.  EA_VIEW_E_WORKER and EA_VIEW_E_SERVER then form it, on the
+ * handle's stream, into one workspace buffer shared by these views, and synchronize the stream
+ * before returning: such a view is a snapshot, valid until the next residual view or the next
+ * round; the kept state is unchanged.  Every other view aliases the live state. */
 enum {
     EA_VIEW_M = 0,             /* worker m (float[d]), Adam at the worker */
     EA_VIEW_V = 1,             /* worker v (float[d]), Adam at the worker */

@@ -44,6 +44,7 @@ struct Layout {
     size_t e_w, m_w, v_w, e_s, m_s, v_s, codes_w, scales_w, codes_s, scales_s, partials;
     size_t off_w, tg_w, pb_w, off_s, tg_s, pb_s, status;
     size_t cuts_w, arr_w, cuts_s, arr_s;  // the grouped pass (groups that span tiles)
+    size_t rview;                         // PASS_LAZY: where a residual view is formed
     int64_t dpad, wcode_stride, wscale_stride;
 };
 
@@ -60,11 +61,14 @@ struct ea_handle {
     float *wscales = nullptr, *sscales = nullptr;
     double *partials = nullptr;
     uint32_t *status = nullptr;
+    float *rview = nullptr;  // PASS_LAZY: the residual views are formed here
     StagePlan splan{};
     Hyper hp{};
     int64_t t = 0;
     uint64_t epoch_w = 0, epoch_s = 0;  // grouped launches so far (worker messages, broadcasts)
     std::vector<unsigned char> compressed;
+    std::vector<unsigned char> lazy_w;  // PASS_LAZY: worker i's e holds its last u (see lazy_residual)
+    bool lazy_s = false;                // PASS_LAZY: e_s holds the last w
     int n_compressed = 0;
     bool has_message = false;
     uint64_t up_bits = 0, down_bits = 0;
@@ -247,6 +251,7 @@ Layout make_layout(const ea_config &c, const QHost &qw, const QHost &qs)
     L.arr_w = gw ? 8 : 0;
     L.cuts_s = gs ? static_cast<size_t>(qs.n_groups + 1) * 8 : 0;
     L.arr_s = gs ? 8 : 0;
+    L.rview = ((gw && qw.kind == EA_Q_SIGN_L1) || (gs && qs.kind == EA_Q_SIGN_L1)) ? vec : 0;
     return L;
 }
 
@@ -254,7 +259,7 @@ size_t layout_bytes(const Layout &L)
 {
     const size_t parts[] = {L.e_w, L.m_w, L.v_w, L.e_s, L.m_s, L.v_s, L.codes_w, L.scales_w, L.codes_s,
                             L.scales_s, L.partials, L.off_w, L.tg_w, L.pb_w, L.off_s, L.tg_s, L.pb_s, L.status,
-                            L.cuts_w, L.arr_w, L.cuts_s, L.arr_s};
+                            L.cuts_w, L.arr_w, L.cuts_s, L.arr_s, L.rview};
     size_t total = 0;
     for (size_t p : parts) total += align_up(p, kAlign);
     return total;
@@ -442,14 +447,20 @@ int check_dev_ptr(ea_handle *h, const void *p, const char *what)
 }
 
 // Finish a message whose scale groups span tiles: scales from the partial norms, then encode.
-int second_pass(ea_handle *h, const QHost &q, float *buf, uint32_t *words, float *scales, uint32_t id)
+// The group scales from the per-(tile, group) partial norms (PASS_STASH, PASS_LAZY).
+int finalize_scales(ea_handle *h, const QHost &q, float *scales)
 {
     FinalizeArgs f{};
     f.d = h->cfg.d;
     f.q = device_quant(q);
     f.partials = h->partials;
     f.scales = scales;
-    int r = check_cuda(h, launch_finalize(f, h->stream), "finalize launch");
+    return check_cuda(h, launch_finalize(f, h->stream), "finalize launch");
+}
+
+int second_pass(ea_handle *h, const QHost &q, float *buf, uint32_t *words, float *scales, uint32_t id)
+{
+    int r = finalize_scales(h, q, scales);
     if (r != EA_OK) return r;
     EncodeArgs e{};
     e.d = h->cfg.d;
@@ -544,6 +555,7 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->stream = static_cast<cudaStream_t>(stream);
     h->n_tiles = (cfg->d + kTile - 1) / kTile;
     h->compressed.assign(cfg->n, 0);
+    h->lazy_w.assign(cfg->n, 0);
     h->hp.alpha = cfg->alpha;
     h->hp.beta1 = cfg->beta1;
     h->hp.beta2 = cfg->beta2;
@@ -580,6 +592,11 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->qw.d_arrive = reinterpret_cast<unsigned long long *>(take(L.arr_w));
     h->qs.d_cuts = reinterpret_cast<int64_t *>(take(L.cuts_s));
     h->qs.d_arrive = reinterpret_cast<unsigned long long *>(take(L.arr_s));
+    h->rview = reinterpret_cast<float *>(take(L.rview));
+    // scaled-sign messages whose groups span tiles: the sign codes need no scale, so one pass writes
+    // them and keeps u (PASS_LAZY); its workspace is that of the two passes
+    if (h->qw.pass == PASS_STASH && h->qw.kind == EA_Q_SIGN_L1) h->qw.pass = PASS_LAZY;
+    if (h->qs.pass == PASS_STASH && h->qs.kind == EA_Q_SIGN_L1) h->qs.pass = PASS_LAZY;
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess) {
@@ -653,6 +670,7 @@ int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
     a.t = static_cast<uint32_t>(h->t);
     a.partials = h->partials;
     a.status = h->status;
+    a.lazy_in = h->qw.pass == PASS_LAZY ? h->lazy_w[worker] : 0;
     if (h->qw.pass == PASS_GROUPED) {
         a.gp = device_group_plan(h->qw, h->epoch_w);
         r = check_cuda(h, launch_worker_grouped(W ? MODE_W : MODE_S, a, h->qw.grid, h->stream), "worker launch");
@@ -661,7 +679,9 @@ int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
         r = check_cuda(h, launch_worker(W ? MODE_W : MODE_S, a, h->stream), "worker launch");
     }
     if (r == EA_OK && h->qw.pass == PASS_STASH) r = second_pass(h, h->qw, a.e, a.words, a.scales, a.id);
+    if (r == EA_OK && h->qw.pass == PASS_LAZY) r = finalize_scales(h, h->qw, a.scales);
     if (r != EA_OK) return r;
+    if (h->qw.pass == PASS_LAZY) h->lazy_w[worker] = h->cfg.error_feedback ? 1 : 0;
     h->compressed[worker] = 1;
     ++h->n_compressed;
     return EA_OK;
@@ -698,9 +718,15 @@ int ea_server_step(ea_handle *h)
     a.wcode_bytes = h->lay.wcode_stride * 4;
     a.status = h->status;
     a.plan = h->splan;
+    a.lazy_in = h->qs.pass == PASS_LAZY && h->lazy_s ? 1 : 0;
     const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
     int r;
-    if (h->qs.pass == PASS_GROUPED) {
+    if (h->qs.pass == PASS_LAZY) {
+        r = check_cuda(h, W ? launch_server_lazy<MODE_W>(a, h->stream) : launch_server_lazy<MODE_S>(a, h->stream),
+                       "server launch");
+        if (r == EA_OK) r = finalize_scales(h, h->qs, h->sscales);
+        if (r == EA_OK) h->lazy_s = h->cfg.error_feedback != 0;
+    } else if (h->qs.pass == PASS_GROUPED) {
         a.gp = device_group_plan(h->qs, h->epoch_s);
         r = check_cuda(h, launch_server_grouped(W ? MODE_W : MODE_S, a, h->qs.grid, h->stream), "server launch");
         if (r == EA_OK) ++h->epoch_s;
@@ -761,7 +787,7 @@ int ea_bits_sent(const ea_handle *h, uint64_t *up_bits, uint64_t *down_bits)
 int ea_round_launches(const ea_handle *h, int32_t *launches)
 {
     if (!h || !launches) return fail(nullptr, EA_E_INVAL, "NULL argument");
-    auto per_message = [](const QHost &q) { return q.pass == PASS_STASH ? 3 : 1; };
+    auto per_message = [](const QHost &q) { return q.pass == PASS_STASH ? 3 : q.pass == PASS_LAZY ? 2 : 1; };
     *launches = h->cfg.n * per_message(h->qw) + per_message(h->qs) + 1;
     return EA_OK;
 }
@@ -789,8 +815,38 @@ int ea_get_view(const ea_handle *h, int32_t which, int32_t index, void **dev_ptr
     switch (which) {
     case EA_VIEW_M: if (W) { p = h->m + index * dp; n = vec; } break;
     case EA_VIEW_V: if (W) { p = h->v + index * dp; n = vec; } break;
-    case EA_VIEW_E_WORKER: p = h->e + index * dp; n = vec; break;
-    case EA_VIEW_E_SERVER: p = h->es; n = vec; break;
+    case EA_VIEW_E_WORKER:
+        p = h->e + index * dp;
+        n = vec;
+        if (h->qw.pass == PASS_LAZY && h->lazy_w[index]) {  // the residual, formed from the kept u
+            ResidArgs ra{};
+            ra.d = h->cfg.d;
+            ra.u = h->e + index * dp;
+            ra.out = h->rview;
+            ra.q = device_quant(h->qw);
+            ra.scales = h->wscales + index * h->lay.wscale_stride;
+            int r = check_cuda(hm, launch_lazy_resid(ra, h->stream), "residual launch");
+            if (r == EA_OK) r = check_cuda(hm, cudaStreamSynchronize(h->stream), "stream synchronize");
+            if (r != EA_OK) return r;
+            p = h->rview;
+        }
+        break;
+    case EA_VIEW_E_SERVER:
+        p = h->es;
+        n = vec;
+        if (h->qs.pass == PASS_LAZY && h->lazy_s) {  // the residual, formed from the kept w
+            ResidArgs ra{};
+            ra.d = h->cfg.d;
+            ra.u = h->es;
+            ra.out = h->rview;
+            ra.q = device_quant(h->qs);
+            ra.scales = h->sscales;
+            int r = check_cuda(hm, launch_lazy_resid(ra, h->stream), "residual launch");
+            if (r == EA_OK) r = check_cuda(hm, cudaStreamSynchronize(h->stream), "stream synchronize");
+            if (r != EA_OK) return r;
+            p = h->rview;
+        }
+        break;
     case EA_VIEW_M_SERVER: if (!W) { p = h->ms; n = vec; } break;
     case EA_VIEW_V_SERVER: if (!W) { p = h->vs; n = vec; } break;
     case EA_VIEW_CODES_WORKER: p = h->wcodes + index * h->lay.wcode_stride; n = h->qw.n_words * 4; break;

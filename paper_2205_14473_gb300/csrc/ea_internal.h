@@ -71,8 +71,12 @@ enum Pass : int {
     PASS_FUSED = 0,   // every group lies inside one tile: reduce, encode and store in one pass
     PASS_STASH = 1,   // groups span tiles: store the input in the residual buffer plus one
                       // partial norm per (tile, group); finalize_kernel and encode_kernel finish
-    PASS_GROUPED = 2  // groups span tiles, one cooperative pass: the input stays in shared memory
+    PASS_GROUPED = 2, // groups span tiles, one cooperative pass: the input stays in shared memory
                       // while the group's partial norms are combined (GroupPlan)
+    PASS_LAZY = 3     // scaled sign, groups span tiles: the codes (signs) need no scale, so one pass
+                      // writes them with the partial norms and keeps u itself in the residual
+                      // buffer; finalize_kernel forms the scales, and e = u - Q(u) is formed from
+                      // (u, s) where it is next needed (the next round's pass, or a view)
 };
 
 // The one-pass plan for scale groups that span tiles.  The vector is cut into waves, coordinate
@@ -114,6 +118,7 @@ struct WorkerArgs {
     double *partials;
     GroupPlan gp;             // PASS_GROUPED
     uint32_t *status;         // device status word (timeouts); may be null outside a handle
+    int lazy_in;              // PASS_LAZY: e holds the previous round's u, scales its scales
 };
 
 // Shared-memory staging plan of the pipelined (persistent, bulk-copy) kernels.  A stage holds one
@@ -151,6 +156,7 @@ struct ServerArgs {
     uint32_t *status;         // device status word (timeouts)
     StagePlan plan;
     GroupPlan gp;             // PASS_GROUPED (Q_s's groups)
+    int lazy_in;              // PASS_LAZY: es holds the previous round's w, scales its scales
 };
 
 // Second pass of PASS_STASH: encode the stashed input in buf, leave the residual in buf.
@@ -172,6 +178,15 @@ struct FinalizeArgs {
     float *scales;
 };
 
+// PASS_LAZY: the residual u - Q(u) of the u kept in `u`, with the scales of its message, into out.
+struct ResidArgs {
+    int64_t d;
+    const float *u;
+    float *out;
+    QParams q;
+    const float *scales;
+};
+
 struct ApplyArgs {
     int64_t d;
     float *x;
@@ -189,6 +204,9 @@ cudaError_t launch_server_grouped_for_qs(const ServerArgs &a, int grid, cudaStre
 template <int MODE, int QS>
 cudaError_t server_grouped_shape_for_qs(int qw, GroupedShape *out);
 cudaError_t launch_server_grouped(int mode, const ServerArgs &a, int grid, cudaStream_t s);
+// PASS_LAZY for a scaled-sign broadcast (instantiated with the QS = QK_SIGN server kernels).
+template <int MODE>
+cudaError_t launch_server_lazy(const ServerArgs &a, cudaStream_t s);
 cudaError_t server_grouped_shape(int mode, int qw, int qs, GroupedShape *out);
 // The server kernel for one placement and broadcast quantizer kind; each (MODE, QS) pair is
 // instantiated only in its own translation unit, ea_server_<mode>_q<QS>.cu.
@@ -199,6 +217,7 @@ cudaError_t launch_server_for_qs(const ServerArgs &a, cudaStream_t s);
 cudaError_t launch_server(int mode, const ServerArgs &a, cudaStream_t s);
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s);
 cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s);
+cudaError_t launch_lazy_resid(const ResidArgs &a, cudaStream_t s);
 cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s);
 cudaError_t launch_fill(float *p, int64_t count, float value, cudaStream_t s);
 

@@ -186,10 +186,12 @@ __global__ void __launch_bounds__(kThreads, 2) server_kernel(const ServerArgs a)
 // Phase one of a grouped server tile: w (the average, after the Adam step with Adam at the server,
 // plus e_s) of the coordinate range [lo, hi) of tile `tile` (0 elsewhere) into ub; m_s and v_s
 // updated and stored in the range.  FULL: the range is the whole tile.
-template <int MODE, int QW, bool FULL>
+template <int MODE, int QW, bool FULL, bool LAZY = false>
 __device__ __forceinline__ void server_u_range(const ServerArgs &a, int64_t tile, int64_t lo, int64_t hi, float4 *ub,
                                                const float *utab, float *stab, TileGroups &tg)
 {
+    LazyScale lzs{};
+    if (LAZY && a.lazy_in) lzs = lazy_scale_of_tile(a.qs, a.scales, tile, a.d);
     float acc[kSlots][4];
     decode_sum_direct<QW>(a, tile, utab, stab, tg, acc);
     const float nf = static_cast<float>(a.n);
@@ -207,6 +209,7 @@ __device__ __forceinline__ void server_u_range(const ServerArgs &a, int64_t tile
                 load4<FULL>(a.ms, q, hi, ms);
                 load4<FULL>(a.vs, q, hi, vs);
             }
+            if (LAZY && a.lazy_in) lazy_residual4<FULL>(a.qs, a.scales, lzs, j0, hi, es);
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -340,7 +343,7 @@ __device__ __forceinline__ void decode_sum_staged(const ServerArgs &a, int64_t t
 // replaces the codes in ub (0 outside the range); m_s, v_s are updated and stored in the range.
 // Returns false, having done nothing, when the tile's scale table would not fit (the caller then
 // takes server_u_range).
-template <int MODE, int QW, bool FULL>
+template <int MODE, int QW, bool FULL, bool LAZY = false>
 __device__ __forceinline__ bool server_u_staged(const ServerArgs &a, int64_t tile, int64_t lo, int64_t hi, float4 *ub,
                                                 const float *utab, float *stab, float *wsc, GroupSmem &gs)
 {
@@ -396,6 +399,14 @@ __device__ __forceinline__ bool server_u_staged(const ServerArgs &a, int64_t til
     float acc[kSlots][4];
     decode_sum_staged<QW>(a, tile, cw, chunk_words, wsc, ngw, gw0, seg, gs.tg, stab, utab, acc);
     compute_sync();  // every thread has read the staged codes
+    if constexpr (LAZY) {
+        if (a.lazy_in) {  // es holds the previous round's w: its residual (lo is the tile's start)
+            const LazyScale lzs = lazy_scale_of_tile(a.qs, a.scales, tile, d);
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k)
+                if (in[k]) lazy_residual4<FULL>(a.qs, a.scales, lzs, 4 * slot_of(tile, k), hi, es[k]);
+        }
+    }
     const float nf = static_cast<float>(n);
     const bool pow2n = (n & (n - 1)) == 0;
     const float inv_n = __frcp_rn(nf);  // exact when n is a power of two
@@ -463,6 +474,65 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_group
     }
 }
 
+
+// PASS_LAZY for a scaled-sign broadcast whose groups span tiles, one CTA per tile.  w (the average,
+// after the Adam step with Adam at the server, plus the residual formed from the previous round's
+// kept w) is stored as the broadcast's signs, which need no scale, and in es as the kept w, with the
+// groups' partial norms; finalize_kernel then forms the broadcast scales.  No CTA waits for another.
+template <int MODE, int QW>
+__global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_lazy_kernel(const ServerArgs a)
+{
+    __shared__ float4 ub[kSlots * kThreads];
+    __shared__ GroupSmem gs;
+    __shared__ float utab_s[256];
+    __shared__ float stab[256];
+    __shared__ float wsc[kWorkerScales];
+    pdl_trigger();
+    const float *utab = build_worker_utab<QW>(a, utab_s);
+    __syncthreads();
+    pdl_wait();
+    const int64_t tile = blockIdx.x;
+    const int64_t d = a.d, lo = tile * kTile, hi = min(lo + static_cast<int64_t>(kTile), d);
+    const bool full = hi == lo + kTile;
+    bool done = false;
+    if (server_codes_fit(a, code_bits<QW>(a.qw)))
+        done = full ? server_u_staged<MODE, QW, true, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs)
+                    : server_u_staged<MODE, QW, false, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs);
+    if (!done) {
+        compute_sync();
+        if (full) server_u_range<MODE, QW, true, true>(a, tile, lo, hi, ub, utab, stab, gs.tg);
+        else server_u_range<MODE, QW, false, true>(a, tile, lo, hi, ub, utab, stab, gs.tg);
+    }
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t qs = slot_of(tile, k);
+        const float4 v = ub[k * kThreads + threadIdx.x];
+        const float w[4] = {v.x, v.y, v.z, v.w};
+        uint32_t c[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float dec;
+            const uint32_t code = encode1<QK_SIGN>(w[i], 0.0f, a.qs, 0.0f, 0, 0.0f, dec);
+            c[i] = (4 * qs + i < d) ? code : 0u;
+        }
+        store_codes4<false, false>(a.words, qs, 1, c, 0, d);
+        if (a.ef && 4 * qs < d) store4(a.es, qs, d, w);
+    }
+    int turn = 0;
+    range_partials<QK_SIGN>(ub, tile, lo, hi, d, a.qs, a.partials, gs, turn);
+}
+
+template <int MODE>
+cudaError_t launch_server_lazy(const ServerArgs &a, cudaStream_t s)
+{
+    const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
+    switch (a.qw.kind) {
+    case QK_SIGN: return launch_pdl(server_lazy_kernel<MODE, QK_SIGN>, grid, block, 0, s, a);
+    case QK_UNIF: return launch_pdl(server_lazy_kernel<MODE, QK_UNIF>, grid, block, 0, s, a);
+    case QK_POW2: return launch_pdl(server_lazy_kernel<MODE, QK_POW2>, grid, block, 0, s, a);
+    default: return launch_pdl(server_lazy_kernel<MODE, QK_IDENT>, grid, block, 0, s, a);
+    }
+}
 
 constexpr int kWorkerTab = 1024;  // floats of the staged server's per-tile worker table
 

@@ -251,13 +251,25 @@ __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64
                                            (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
             return;
         }
-        // PASS_STASH
+        // PASS_STASH: u into resid for encode_kernel.  PASS_LAZY (scaled sign): u into resid, where
+        // the residual is formed from it and the scale later (lazy_residual; without error feedback
+        // the residual stays 0), and the codes now: the sign of u needs no scale.
 #pragma unroll
         for (int k = 0; k < kSlots; ++k) {
             const int64_t qs = slot_of(tile, k);
             float uk[4];
             src.get(k, uk);
-            if (FULL || 4 * qs < d) store4<FULL>(resid, qs, d, uk);
+            if ((PASS != PASS_LAZY || ef) && (FULL || 4 * qs < d)) store4<FULL>(resid, qs, d, uk);
+            if constexpr (PASS == PASS_LAZY && QK == QK_SIGN) {
+                uint32_t c[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    float dec;
+                    const uint32_t code = encode1<QK>(uk[i], 0.0f, q, 0.0f, 0, 0.0f, dec);
+                    c[i] = (FULL || 4 * qs + i < d) ? code : 0u;
+                }
+                store_codes4<FULL, BALLOT>(words, qs, 1, c, 0, d);
+            }
         }
         const Grouping &G = q.grp;
         for (int64_t gi = first_group_of_tile(G, tile);; ++gi) {
@@ -293,6 +305,51 @@ __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64
             if (ge >= tile_hi) break;
         }
     }
+}
+
+// PASS_LAZY (scaled sign): where the residual e = u - Q(u) of a kept u is formed -- u - (u >= 0 ? s
+// : -s), s the scale of the coordinate's group in the previous message (scales).  This is
+// e <- u - Q(u) of Algorithm 1 / Algorithm 2 with the same binary32 operations, evaluated where the
+// residual is next read.  LazyScale holds a tile's scale when the tile lies in one group (loaded
+// once, early), else the group to start the per-coordinate lookups from.
+struct LazyScale {
+    int64_t g1, hint;  // the tile's one group (-1: several), the tile's first group
+    float s1;          // the scale of g1
+};
+
+__device__ __forceinline__ LazyScale lazy_scale_of_tile(const QParams &q, const float *scales, int64_t tile, int64_t d)
+{
+    LazyScale ls;
+    ls.g1 = tile_single_group(q.grp, tile, d);
+    ls.hint = first_group_of_tile(q.grp, tile);
+    ls.s1 = ls.g1 >= 0 ? scales[ls.g1] : 0.0f;
+    return ls;
+}
+
+// The residual of the kept u of coordinates j0 .. j0+3 (in place in e); coordinates >= d unchanged.
+template <bool FULL>
+__device__ __forceinline__ void lazy_residual4(const QParams &q, const float *scales, const LazyScale &ls, int64_t j0,
+                                               int64_t d, float (&e)[4])
+{
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        if (FULL || j0 + i < d) {
+            const float s = ls.g1 >= 0 ? ls.s1 : scales[group_of(q.grp, j0 + i, ls.hint)];
+            float dec;
+            (void)encode1<QK_SIGN>(e[i], s, q, 0.0f, 0, 0.0f, dec);
+            e[i] = __fsub_rn(e[i], dec);
+        }
+    }
+}
+
+// The same for all of this thread's slots of tile `tile`.
+template <bool FULL>
+__device__ __forceinline__ void lazy_residual(const QParams &q, const float *scales, int64_t tile, int64_t d,
+                                              float (&e)[kSlots][4])
+{
+    const LazyScale ls = lazy_scale_of_tile(q, scales, tile, d);
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) lazy_residual4<FULL>(q, scales, ls, 4 * slot_of(tile, k), d, e[k]);
 }
 
 }  // namespace ea

@@ -24,6 +24,10 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
     // the grid's fl(i/L) table, built while the loads are in flight (read after the scale
     // reduction's barrier)
     build_qtab<QK>(a.q, sm.qtab);
+    if constexpr (PASS == PASS_LAZY) {
+        // e holds the previous round's u: its residual is u - Q(u) with the previous scales
+        if (a.lazy_in) lazy_residual<FULL>(a.q, a.scales, tile, d, e);
+    }
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
         const int64_t q = slot_of(tile, k);
@@ -53,6 +57,21 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
 // coordinate), three with Adam at the worker.  Measured: the server-side-Adam uniform grid runs
 // faster at four CTAs with a few bytes of spill than at three without, and the worker-side-Adam
 // uniform grid faster at three (80 registers, a few bytes of spill) than at two.
+// PASS_LAZY for the scaled sign: the same tile, the codes stored with the partial norms and u kept
+// in e (see lazy_residual); one launch per message plus finalize_kernel.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 3)
+    worker_lazy_kernel(const WorkerArgs a)
+{
+    __shared__ TileSmem sm;
+    __shared__ float4 ubuf[kSlots * kThreads];
+    pdl_trigger();
+    pdl_wait();
+    const int64_t tile = blockIdx.x;
+    if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK_SIGN, true, PASS_LAZY>(a, tile, ubuf, sm);
+    else worker_tile<MODE, QK_SIGN, false, PASS_LAZY>(a, tile, ubuf, sm);
+}
+
 template <int MODE, int QK>
 __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 3)
     worker_kernel(const WorkerArgs a)
@@ -356,6 +375,8 @@ template <int MODE>
 static cudaError_t launch_worker_mode(const WorkerArgs &a, cudaStream_t s)
 {
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
+    if (a.pass == PASS_LAZY)
+        return a.q.kind == QK_SIGN ? launch_pdl(worker_lazy_kernel<MODE>, grid, block, 0, s, a) : cudaErrorNotSupported;
     switch (a.q.kind) {
     case QK_SIGN: return launch_pdl(worker_kernel<MODE, QK_SIGN>, grid, block, 0, s, a);
     case QK_UNIF: return launch_pdl(worker_kernel<MODE, QK_UNIF>, grid, block, 0, s, a);
@@ -402,6 +423,30 @@ cudaError_t launch_encode(const EncodeArgs &a, cudaStream_t s)
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
     if (a.q.kind == QK_SIGN) return launch_pdl(encode_kernel<QK_SIGN>, grid, block, 0, s, a);
     return launch_pdl(encode_kernel<QK_UNIF>, grid, block, 0, s, a);
+}
+
+// The residual u - Q(u) of the u kept by PASS_LAZY, into a.out, one CTA per tile (a view of it).
+__global__ void __launch_bounds__(kThreads) lazy_resid_kernel(const ResidArgs a)
+{
+    pdl_trigger();
+    pdl_wait();
+    const int64_t tile = blockIdx.x;
+    const bool full = (tile + 1) * kTile <= a.d;
+    float u[kSlots][4];
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) load4(a.u, slot_of(tile, k), a.d, u[k]);
+    if (full) lazy_residual<true>(a.q, a.scales, tile, a.d, u);
+    else lazy_residual<false>(a.q, a.scales, tile, a.d, u);
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k)
+        if (4 * slot_of(tile, k) < a.d) store4(a.out, slot_of(tile, k), a.d, u[k]);
+}
+
+cudaError_t launch_lazy_resid(const ResidArgs &a, cudaStream_t s)
+{
+    const dim3 grid(static_cast<unsigned>((a.d + kTile - 1) / kTile)), block(kThreads);
+    if (a.q.kind != QK_SIGN) return cudaErrorNotSupported;
+    return launch_pdl(lazy_resid_kernel, grid, block, 0, s, a);
 }
 
 cudaError_t launch_apply(const ApplyArgs &a, cudaStream_t s)

@@ -42,6 +42,8 @@ def test_workspace_bytes_covers_state(ea_lib):
             c, keep = cfg.to_c()
             nbytes = ea.ea_workspace_bytes(c)
             vecs = (3 * w.n + 1) if placement == ea.ADAM_AT_WORKER else (w.n + 3)
+            # scaled-sign worker groups that span tiles: one more vector, where residual views are formed
+            vecs += int(w.qw.kind == W.Q_SIGN_L1 and w.qw.group <= 0 and w.d > 4096)
             code_bytes = (w.n * w.d * w.qw.bits + w.d * w.qs.bits) / 8
             assert nbytes >= vecs * w.d * 4 + code_bytes
             assert nbytes <= (vecs * w.d * 4 + code_bytes) * 1.01 + 2**22, name

@@ -133,36 +133,44 @@ def test_staged_server_several_tiles_per_cta(qw, qs, placement):
 
 def test_two_pass_scale_beyond_the_grouped_capacity():
     """A whole-vector scale over 12.3 million coordinates: more tiles than the one-pass grouped
-    kernels hold in shared memory at once (about 1,800 on a GB300), so both messages take the
-    two-pass scale (stash, finalize, encode: three launches each)."""
+    kernels hold in shared memory at once (about 1,800 on a GB300).  The uniform-grid broadcast
+    takes the two-pass scale (stash, finalize, encode: three launches); the scaled-sign worker
+    messages take the lazy pass (codes with the partial norms, then finalize: two launches)."""
     d = 3000 * 4096 + 3
     cfg = ea.EAConfig(d=d, n=2, qw=W.sign_q(0), qs=W.uniform_q(8, 0, False), alpha=1e-3, seed=41)
-    L = _run_host(cfg, 2, seed=43)
-    assert L.gpu.launches_per_round == 2 * 3 + 3 + 1
+    L = _run_host(cfg, 3, seed=43)
+    assert L.gpu.launches_per_round == 2 * 2 + 3 + 1
 
 
-@pytest.mark.parametrize("qw,qs", [(W.sign_q(0), W.sign_q(0)), (W.uniform_q(4, 0, True), W.uniform_q(8, 1000, False))])
-def test_grouped_scales_one_launch_per_message(qw, qs):
-    """Scale groups that span tiles take the one-pass grouped kernels (74 tiles: one per worker CTA):
-    one launch per message."""
+@pytest.mark.parametrize("qw,qs,launches", [(W.sign_q(0), W.sign_q(0), 3 * 2 + 2 + 1),
+                                           (W.uniform_q(4, 0, True), W.uniform_q(8, 1000, False), 3 * 1 + 1 + 1)])
+def test_grouped_scales_one_launch_per_message(qw, qs, launches):
+    """Scale groups that span tiles (74 tiles): uniform-grid messages take the one-pass grouped
+    kernels (one tile per worker CTA, one launch each); scaled-sign messages take the lazy pass (the
+    signs with the partial norms, then finalize: two launches each)."""
     cfg = ea.EAConfig(d=300_001, n=3, qw=qw, qs=qs, alpha=1e-3, seed=45)
     L = _run_host(cfg, 3, seed=47)
-    assert L.gpu.launches_per_round == 3 + 1 + 1
+    assert L.gpu.launches_per_round == launches
 
 
-@pytest.mark.parametrize("qw,qs,placement", [
-    (W.sign_q(0), W.sign_q(0), ea.ADAM_AT_WORKER),
-    (W.uniform_q(4, 0, True), W.uniform_q(8, 0, False), ea.ADAM_AT_SERVER),
+@pytest.mark.parametrize("qw,qs,placement,launches", [
+    (W.sign_q(0), W.sign_q(0), ea.ADAM_AT_WORKER, 3 * 2 + 2 + 1),
+    (W.uniform_q(4, 0, True), W.uniform_q(8, 0, False), ea.ADAM_AT_SERVER, 3 * 3 + 1 + 1),
+    (W.uniform_q(4, 0, True), W.uniform_q(8, 0, False), ea.ADAM_AT_WORKER, 3 * 3 + 1 + 1),
     (W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)), W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)),
-     ea.ADAM_AT_WORKER),
+     ea.ADAM_AT_WORKER, 3 * 2 + 2 + 1),
+    (W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)), W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)),
+     ea.ADAM_AT_SERVER, 3 * 2 + 2 + 1),
 ])
-def test_grouped_broadcast_with_several_tiles_per_cta(qw, qs, placement):
-    """4.4 million coordinates (1,075 tiles): the grouped broadcast's CTAs each hold several tiles
-    of one wave, while the workers' messages take the two-pass scale."""
+def test_grouped_broadcast_with_several_tiles_per_cta(qw, qs, placement, launches):
+    """4.4 million coordinates (1,075 tiles).  A uniform-grid broadcast takes the grouped kernel,
+    whose CTAs each hold several tiles of one wave, and the worker messages the two-pass scale; a
+    scaled-sign broadcast and scaled-sign worker messages take the lazy pass (whole vector, and
+    segments with tiles that hold several groups)."""
     d = 4_400_200
     cfg = ea.EAConfig(d=d, n=3, qw=qw, qs=qs, alpha=1e-3, placement=placement, seed=49)
-    L = _run_host(cfg, 2, seed=51)
-    assert L.gpu.launches_per_round == 3 * 3 + 1 + 1
+    L = _run_host(cfg, 3, seed=51)
+    assert L.gpu.launches_per_round == launches
 
 
 def test_replicas_are_identical_and_protocol():
@@ -215,7 +223,7 @@ def test_c1_full():
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
     assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (2_622_720, 2_622_720)
-    assert L.gpu.launches_per_round == w.n + 2  # whole-vector scales in one pass per message
+    assert L.gpu.launches_per_round == 2 * w.n + 2 + 1  # scaled-sign messages: the lazy pass + finalize
 
 
 def test_c2_quadratic_toy_full():
@@ -256,8 +264,8 @@ def test_c3_resnet18_all_tensors(placement, rounds):
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
     assert L.total_mismatch == 0
-    # per-tensor scales: the broadcast in one grouped pass; the 2,854-tile worker messages in two
-    assert L.gpu.launches_per_round == 3 * w.n + 2
+    # per-tensor scales: every message in the lazy pass (codes and partial norms, then finalize)
+    assert L.gpu.launches_per_round == 2 * w.n + 2 + 1
     if rounds == w.rounds:
         assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (18_706_393_600, 18_706_393_600)
 
