@@ -69,6 +69,7 @@ struct ea_handle {
     std::vector<unsigned char> compressed;
     std::vector<unsigned char> lazy_w;  // PASS_LAZY: worker i's e holds its last u (see lazy_residual)
     bool lazy_s = false;                // PASS_LAZY: e_s holds the last w
+    bool lazy_staged = false;           // PASS_LAZY broadcast: every tile's worker messages fit the staging
     int n_compressed = 0;
     bool has_message = false;
     uint64_t up_bits = 0, down_bits = 0;
@@ -345,6 +346,22 @@ void try_grouped(QHost &q, int64_t d, int64_t n_tiles, const GroupedShape &shape
     q.pass = PASS_GROUPED;
 }
 
+// The most of q's scale groups that meet one 4096-tile.
+int64_t max_groups_per_tile(const QHost &q, int64_t d, int64_t n_tiles)
+{
+    if (!q.has_scales || q.gkind == GK_WHOLE) return 1;
+    if (q.gkind == GK_BLOCK) return (kTile - 1) / q.G + 2;  // a bound
+    int64_t most = 1;
+    for (int64_t t = 0; t < n_tiles; ++t) {
+        const int64_t last = std::min((t + 1) * kTile, d) - 1;
+        const int64_t g0 = q.tile_group[static_cast<size_t>(t)];
+        int64_t g = g0;
+        while (q.offsets[static_cast<size_t>(g + 1)] <= last) ++g;
+        most = std::max(most, g - g0 + 1);
+    }
+    return most;
+}
+
 GroupPlan device_group_plan(const QHost &q, uint64_t epoch)
 {
     GroupPlan g{};
@@ -498,23 +515,19 @@ cudaError_t ea::launch_server(int mode, const ServerArgs &a, cudaStream_t s)
     }
 }
 
+// The grouped server exists for a uniform-grid broadcast (a scaled-sign one takes PASS_LAZY).
 cudaError_t ea::launch_server_grouped(int mode, const ServerArgs &a, int grid, cudaStream_t s)
 {
-    if (mode == MODE_W)
-        return a.qs.kind == QK_SIGN ? launch_server_grouped_for_qs<MODE_W, QK_SIGN>(a, grid, s)
-                                    : launch_server_grouped_for_qs<MODE_W, QK_UNIF>(a, grid, s);
-    return a.qs.kind == QK_SIGN ? launch_server_grouped_for_qs<MODE_S, QK_SIGN>(a, grid, s)
-                                : launch_server_grouped_for_qs<MODE_S, QK_UNIF>(a, grid, s);
+    if (a.qs.kind != QK_UNIF) return cudaErrorNotSupported;
+    return mode == MODE_W ? launch_server_grouped_for_qs<MODE_W, QK_UNIF>(a, grid, s)
+                          : launch_server_grouped_for_qs<MODE_S, QK_UNIF>(a, grid, s);
 }
 
 cudaError_t ea::server_grouped_shape(int mode, int qw, int qs, GroupedShape *out)
 {
-    if (qs != QK_SIGN && qs != QK_UNIF) return cudaErrorNotSupported;
-    if (mode == MODE_W)
-        return qs == QK_SIGN ? server_grouped_shape_for_qs<MODE_W, QK_SIGN>(qw, out)
-                             : server_grouped_shape_for_qs<MODE_W, QK_UNIF>(qw, out);
-    return qs == QK_SIGN ? server_grouped_shape_for_qs<MODE_S, QK_SIGN>(qw, out)
-                         : server_grouped_shape_for_qs<MODE_S, QK_UNIF>(qw, out);
+    if (qs != QK_UNIF) return cudaErrorNotSupported;
+    return mode == MODE_W ? server_grouped_shape_for_qs<MODE_W, QK_UNIF>(qw, out)
+                          : server_grouped_shape_for_qs<MODE_S, QK_UNIF>(qw, out);
 }
 
 extern "C" {
@@ -596,7 +609,13 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     // scaled-sign messages whose groups span tiles: the sign codes need no scale, so one pass writes
     // them and keeps u (PASS_LAZY); its workspace is that of the two passes
     if (h->qw.pass == PASS_STASH && h->qw.kind == EA_Q_SIGN_L1) h->qw.pass = PASS_LAZY;
-    if (h->qs.pass == PASS_STASH && h->qs.kind == EA_Q_SIGN_L1) h->qs.pass = PASS_LAZY;
+    if (h->qs.pass == PASS_STASH && h->qs.kind == EA_Q_SIGN_L1) {
+        h->qs.pass = PASS_LAZY;
+        // the server stages a tile's worker codes and scales in shared memory when they fit
+        const int64_t g = max_groups_per_tile(h->qw, cfg->d, h->n_tiles);
+        h->lazy_staged = static_cast<int64_t>(cfg->n) * h->qw.bits <= 32 &&
+                         g <= kStagedTileGroups && cfg->n * g <= kWorkerScales;
+    }
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess) {
@@ -722,7 +741,8 @@ int ea_server_step(ea_handle *h)
     const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
     int r;
     if (h->qs.pass == PASS_LAZY) {
-        r = check_cuda(h, W ? launch_server_lazy<MODE_W>(a, h->stream) : launch_server_lazy<MODE_S>(a, h->stream),
+        r = check_cuda(h, W ? launch_server_lazy<MODE_W>(a, h->lazy_staged, h->stream)
+                            : launch_server_lazy<MODE_S>(a, h->lazy_staged, h->stream),
                        "server launch");
         if (r == EA_OK) r = finalize_scales(h, h->qs, h->sscales);
         if (r == EA_OK) h->lazy_s = h->cfg.error_feedback != 0;

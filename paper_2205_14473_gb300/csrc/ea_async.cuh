@@ -14,6 +14,7 @@
 namespace ea {
 
 constexpr uint32_t kStatusTimeout = 1u;
+constexpr uint32_t kStatusCheck = 2u;  // a kernel found an input outside what its launch assumed
 constexpr long long kWaitLimitCycles = 4000000000LL;  // ~2 s at the 2.07 GHz SM clock
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)

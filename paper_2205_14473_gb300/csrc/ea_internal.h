@@ -21,6 +21,10 @@ constexpr uint32_t kServerMaxDynSmem = 200 * 1024;
 constexpr uint32_t kSmemPerSm = 228 * 1024;
 constexpr uint32_t kSmemReservedPerCta = 1024;
 constexpr int kWarps = kThreads / 32;
+// Shared-memory staging of a server tile's worker scales: at most kStagedTileGroups of Q_w's groups
+// meet one tile, and n times that many scales fit in kWorkerScales.
+constexpr int kWorkerScales = 512;
+constexpr int kStagedTileGroups = 256;
 // Device ordinals for which per-device host state (kernel attributes) is kept.
 constexpr int kMaxDevices = 64;
 
@@ -205,8 +209,9 @@ template <int MODE, int QS>
 cudaError_t server_grouped_shape_for_qs(int qw, GroupedShape *out);
 cudaError_t launch_server_grouped(int mode, const ServerArgs &a, int grid, cudaStream_t s);
 // PASS_LAZY for a scaled-sign broadcast (instantiated with the QS = QK_SIGN server kernels).
+// staged: every tile's worker codes and scales fit the shared-memory staging (lazy_server_staged).
 template <int MODE>
-cudaError_t launch_server_lazy(const ServerArgs &a, cudaStream_t s);
+cudaError_t launch_server_lazy(const ServerArgs &a, bool staged, cudaStream_t s);
 cudaError_t server_grouped_shape(int mode, int qw, int qs, GroupedShape *out);
 // The server kernel for one placement and broadcast quantizer kind; each (MODE, QS) pair is
 // instantiated only in its own translation unit, ea_server_<mode>_q<QS>.cu.

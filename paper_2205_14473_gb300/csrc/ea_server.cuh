@@ -249,7 +249,6 @@ __device__ __forceinline__ void load_codes4_smem(const uint32_t *words, int ls, 
     }
 }
 
-constexpr int kWorkerScales = 512;  // worker scales of a tile's groups held by the grouped server
 
 // Whether the grouped server stages a tile's worker codes in shared memory: all n chunks must fit
 // in the tile's slot (4096 b_w / 8 bytes each, 16 KB in all).
@@ -318,6 +317,25 @@ __device__ __forceinline__ void decode_sum_staged(const ServerArgs &a, int64_t t
             }
         }
     }
+    if constexpr (QW == QK_SIGN) {
+        if (ngw == 1) {
+            // the workers past the table, in order: each one's sign nibble of the slot, then a
+            // select of +-s_w and one addition per coordinate
+#pragma unroll 1
+            for (int w = w_first; w < n; ++w) {
+                const uint32_t *ww = cw + w * chunk_words;
+                const float sw = wsc[w], nsw = -sw;
+#pragma unroll
+                for (int k = 0; k < kSlots; ++k) {
+                    const int ls = k * kThreads + threadIdx.x;
+                    const uint32_t nib = ww[ls >> 3] >> (4 * (ls & 7));
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) acc[k][i] = __fadd_rn(acc[k][i], ((nib >> i) & 1u) ? sw : nsw);
+                }
+            }
+            return;
+        }
+    }
 #pragma unroll 1
     for (int w = w_first; w < n; ++w) {
         const uint32_t *ww = cw + w * chunk_words;
@@ -357,7 +375,7 @@ __device__ __forceinline__ bool server_u_staged(const ServerArgs &a, int64_t til
         gw0 = first_group_of_tile(GW, tile);
         const int64_t last = min(tile * kTile + static_cast<int64_t>(kTile), d) - 1;
         ngw = static_cast<int>(group_of(GW, last, gw0) - gw0 + 1);
-        if (n * ngw > kWorkerScales || ngw > 256) return false;
+        if (n * ngw > kWorkerScales || ngw > kStagedTileGroups) return false;
     }
     const bool seg = has_scale<QW>() && ngw > 1 && GW.gkind == GK_SEG;
     float es[kSlots][4], ms[kSlots][4], vs[kSlots][4];
@@ -479,7 +497,9 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_group
 // after the Adam step with Adam at the server, plus the residual formed from the previous round's
 // kept w) is stored as the broadcast's signs, which need no scale, and in es as the kept w, with the
 // groups' partial norms; finalize_kernel then forms the broadcast scales.  No CTA waits for another.
-template <int MODE, int QW>
+// STAGED: every tile's worker codes and scales fit the shared-memory staging (the host checks
+// server_codes_fit and the groups per tile), and only that path is compiled in; else direct loads.
+template <int MODE, int QW, bool STAGED>
 __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_lazy_kernel(const ServerArgs a)
 {
     __shared__ float4 ub[kSlots * kThreads];
@@ -494,12 +514,14 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_lazy_
     const int64_t tile = blockIdx.x;
     const int64_t d = a.d, lo = tile * kTile, hi = min(lo + static_cast<int64_t>(kTile), d);
     const bool full = hi == lo + kTile;
-    bool done = false;
-    if (server_codes_fit(a, code_bits<QW>(a.qw)))
-        done = full ? server_u_staged<MODE, QW, true, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs)
-                    : server_u_staged<MODE, QW, false, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs);
-    if (!done) {
-        compute_sync();
+    if constexpr (STAGED) {
+        const bool done = full ? server_u_staged<MODE, QW, true, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs)
+                               : server_u_staged<MODE, QW, false, true>(a, tile, lo, hi, ub, utab, stab, wsc, gs);
+        if (!done) {  // outside what the host checked: report it, store nothing
+            if (threadIdx.x == 0) report_status(a.status, kStatusCheck);
+            return;
+        }
+    } else {
         if (full) server_u_range<MODE, QW, true, true>(a, tile, lo, hi, ub, utab, stab, gs.tg);
         else server_u_range<MODE, QW, false, true>(a, tile, lo, hi, ub, utab, stab, gs.tg);
     }
@@ -522,16 +544,22 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 2 : 3) server_lazy_
     range_partials<QK_SIGN>(ub, tile, lo, hi, d, a.qs, a.partials, gs, turn);
 }
 
-template <int MODE>
-cudaError_t launch_server_lazy(const ServerArgs &a, cudaStream_t s)
+template <int MODE, bool STAGED>
+static cudaError_t launch_server_lazy_st(const ServerArgs &a, cudaStream_t s)
 {
     const dim3 grid(static_cast<unsigned>(a.n_tiles)), block(kThreads);
     switch (a.qw.kind) {
-    case QK_SIGN: return launch_pdl(server_lazy_kernel<MODE, QK_SIGN>, grid, block, 0, s, a);
-    case QK_UNIF: return launch_pdl(server_lazy_kernel<MODE, QK_UNIF>, grid, block, 0, s, a);
-    case QK_POW2: return launch_pdl(server_lazy_kernel<MODE, QK_POW2>, grid, block, 0, s, a);
-    default: return launch_pdl(server_lazy_kernel<MODE, QK_IDENT>, grid, block, 0, s, a);
+    case QK_SIGN: return launch_pdl(server_lazy_kernel<MODE, QK_SIGN, STAGED>, grid, block, 0, s, a);
+    case QK_UNIF: return launch_pdl(server_lazy_kernel<MODE, QK_UNIF, STAGED>, grid, block, 0, s, a);
+    case QK_POW2: return launch_pdl(server_lazy_kernel<MODE, QK_POW2, STAGED>, grid, block, 0, s, a);
+    default: return launch_pdl(server_lazy_kernel<MODE, QK_IDENT, STAGED>, grid, block, 0, s, a);
     }
+}
+
+template <int MODE>
+cudaError_t launch_server_lazy(const ServerArgs &a, bool staged, cudaStream_t s)
+{
+    return staged ? launch_server_lazy_st<MODE, true>(a, s) : launch_server_lazy_st<MODE, false>(a, s);
 }
 
 constexpr int kWorkerTab = 1024;  // floats of the staged server's per-tile worker table
@@ -950,11 +978,11 @@ static cudaError_t launch_server_staged(const ServerArgs &a, cudaStream_t s)
 }
 
 
-// The grouped server for one placement and broadcast kind (Q_s with scale groups only).
+// The grouped server for one placement and broadcast kind (the uniform grid only).
 template <int MODE, int QS>
 cudaError_t server_grouped_shape_for_qs(int qw, GroupedShape *out)
 {
-    if constexpr (QS != QK_SIGN && QS != QK_UNIF) {
+    if constexpr (QS != QK_UNIF) {
         return cudaErrorNotSupported;
     } else {
         const int w = MODE == MODE_S ? 2 : 3;  // the kernel's launch bounds
@@ -970,7 +998,7 @@ cudaError_t server_grouped_shape_for_qs(int qw, GroupedShape *out)
 template <int MODE, int QS>
 cudaError_t launch_server_grouped_for_qs(const ServerArgs &a, int grid, cudaStream_t s)
 {
-    if constexpr (QS != QK_SIGN && QS != QK_UNIF) {
+    if constexpr (QS != QK_UNIF) {
         return cudaErrorNotSupported;
     } else {
         const int slots = a.gp.slots;

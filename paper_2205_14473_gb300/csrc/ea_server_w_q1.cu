@@ -3,7 +3,5 @@
 
 namespace ea {
 template cudaError_t launch_server_for_qs<MODE_W, QK_SIGN>(const ServerArgs &, cudaStream_t);
-template cudaError_t launch_server_grouped_for_qs<MODE_W, QK_SIGN>(const ServerArgs &, int, cudaStream_t);
-template cudaError_t server_grouped_shape_for_qs<MODE_W, QK_SIGN>(int, GroupedShape *);
-template cudaError_t launch_server_lazy<MODE_W>(const ServerArgs &, cudaStream_t);
+template cudaError_t launch_server_lazy<MODE_W>(const ServerArgs &, bool, cudaStream_t);
 }  // namespace ea

@@ -202,6 +202,10 @@ __device__ __forceinline__ void finish_tile_smem(const float4 *ubuf, DF l1, floa
                                    (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
 }
 
+// PASS_LAZY on a tile that lies inside one scale group: a compile-time refinement of the pass
+// (one partial norm, no per-coordinate group bounds), chosen per tile by the lazy kernels.
+constexpr int PASS_LAZY_ONE = 16;
+
 // The tile's end for a quantizer with scale groups, u read through `src` (URegs or USmem).
 //   PASS_FUSED: the tile is exactly one scale group (blocks of 4096): reduce, encode, store.
 //   PASS_STASH: store u in resid and one partial norm per (tile, group) for finalize/encode.
@@ -249,6 +253,34 @@ __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64
             // sm.qtab was filled by build_qtab before the reduction's barrier
             encode_store<QK, FULL, BALLOT>(src, s, tile, d, q, words, resid, ef, seed, id, t,
                                            (QK == QK_UNIF && q.bits <= 8) ? sm.qtab : nullptr);
+            return;
+        }
+        if constexpr (PASS == PASS_LAZY_ONE && QK == QK_SIGN) {
+            // u (with error feedback), the codes, and the one group's partial norm of the tile --
+            // the same sum, in the same order, as the per-group loop below forms
+            DF acc{0.0f, 0.0f};
+#pragma unroll
+            for (int k = 0; k < kSlots; ++k) {
+                const int64_t qs = slot_of(tile, k);
+                float uk[4];
+                src.get(k, uk);
+                if (ef && (FULL || 4 * qs < d)) store4<FULL>(resid, qs, d, uk);
+                uint32_t c[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    float dec;
+                    const uint32_t code = encode1<QK>(uk[i], 0.0f, q, 0.0f, 0, 0.0f, dec);
+                    c[i] = (FULL || 4 * qs + i < d) ? code : 0u;
+                    df_accumulate(acc, fabsf(uk[i]));  // u beyond d is 0
+                }
+                store_codes4<FULL, BALLOT>(words, qs, 1, c, 0, d);
+            }
+            const double part = block_sum(acc, sm.red, &sm.bcast);
+            if (threadIdx.x == 0) {
+                const Grouping &G = q.grp;
+                const int64_t g = first_group_of_tile(G, tile);
+                partials[G.pair_base[g] + (tile - group_begin(G, g, d) / kTile)] = part;
+            }
             return;
         }
         // PASS_STASH: u into resid for encode_kernel.  PASS_LAZY (scaled sign): u into resid, where
@@ -343,10 +375,27 @@ __device__ __forceinline__ void lazy_residual4(const QParams &q, const float *sc
 }
 
 // The same for all of this thread's slots of tile `tile`.
-template <bool FULL>
+// ONE: the tile lies inside one group (no per-coordinate lookups are compiled in).
+template <bool FULL, bool ONE = false>
 __device__ __forceinline__ void lazy_residual(const QParams &q, const float *scales, int64_t tile, int64_t d,
                                               float (&e)[kSlots][4])
 {
+    if constexpr (ONE) {
+        const float s = scales[first_group_of_tile(q.grp, tile)];
+#pragma unroll
+        for (int k = 0; k < kSlots; ++k) {
+            const int64_t j0 = 4 * slot_of(tile, k);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                if (FULL || j0 + i < d) {
+                    float dec;
+                    (void)encode1<QK_SIGN>(e[k][i], s, q, 0.0f, 0, 0.0f, dec);
+                    e[k][i] = __fsub_rn(e[k][i], dec);
+                }
+            }
+        }
+        return;
+    }
     const LazyScale ls = lazy_scale_of_tile(q, scales, tile, d);
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) lazy_residual4<FULL>(q, scales, ls, 4 * slot_of(tile, k), d, e[k]);

@@ -24,9 +24,9 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
     // the grid's fl(i/L) table, built while the loads are in flight (read after the scale
     // reduction's barrier)
     build_qtab<QK>(a.q, sm.qtab);
-    if constexpr (PASS == PASS_LAZY) {
+    if constexpr (PASS == PASS_LAZY || PASS == PASS_LAZY_ONE) {
         // e holds the previous round's u: its residual is u - Q(u) with the previous scales
-        if (a.lazy_in) lazy_residual<FULL>(a.q, a.scales, tile, d, e);
+        if (a.lazy_in) lazy_residual<FULL, PASS == PASS_LAZY_ONE>(a.q, a.scales, tile, d, e);
     }
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
@@ -68,8 +68,12 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 3)
     pdl_trigger();
     pdl_wait();
     const int64_t tile = blockIdx.x;
-    if ((tile + 1) * kTile <= a.d) worker_tile<MODE, QK_SIGN, true, PASS_LAZY>(a, tile, ubuf, sm);
-    else worker_tile<MODE, QK_SIGN, false, PASS_LAZY>(a, tile, ubuf, sm);
+    if ((tile + 1) * kTile <= a.d) {
+        if (tile_single_group(a.q.grp, tile, a.d) >= 0) worker_tile<MODE, QK_SIGN, true, PASS_LAZY_ONE>(a, tile, ubuf, sm);
+        else worker_tile<MODE, QK_SIGN, true, PASS_LAZY>(a, tile, ubuf, sm);
+    } else {
+        worker_tile<MODE, QK_SIGN, false, PASS_LAZY>(a, tile, ubuf, sm);
+    }
 }
 
 template <int MODE, int QK>
@@ -390,25 +394,21 @@ cudaError_t launch_worker(int mode, const WorkerArgs &a, cudaStream_t s)
     return mode == MODE_W ? launch_worker_mode<MODE_W>(a, s) : launch_worker_mode<MODE_S>(a, s);
 }
 
-// The grouped kernels exist for the quantizers with scale groups (scaled sign, uniform grid).
+// The grouped kernel exists for the uniform grid (a scaled-sign message takes PASS_LAZY).
 cudaError_t worker_grouped_shape(int mode, int qk, GroupedShape *out)
 {
     const int w = mode == MODE_W ? 2 : 4;  // the kernels' launch bounds
-    if (mode == MODE_W && qk == QK_SIGN) return grouped_shape(worker_grouped_kernel<MODE_W, QK_SIGN>, w, out);
-    if (mode == MODE_W && qk == QK_UNIF) return grouped_shape(worker_grouped_kernel<MODE_W, QK_UNIF>, w, out);
-    if (mode == MODE_S && qk == QK_SIGN) return grouped_shape(worker_grouped_kernel<MODE_S, QK_SIGN>, w, out);
-    if (mode == MODE_S && qk == QK_UNIF) return grouped_shape(worker_grouped_kernel<MODE_S, QK_UNIF>, w, out);
-    return cudaErrorNotSupported;
+    if (qk != QK_UNIF) return cudaErrorNotSupported;
+    return mode == MODE_W ? grouped_shape(worker_grouped_kernel<MODE_W, QK_UNIF>, w, out)
+                          : grouped_shape(worker_grouped_kernel<MODE_S, QK_UNIF>, w, out);
 }
 
 cudaError_t launch_worker_grouped(int mode, const WorkerArgs &a, int grid, cudaStream_t s)
 {
     const int slots = a.gp.slots;
-    if (mode == MODE_W && a.q.kind == QK_SIGN) return grouped_launch(worker_grouped_kernel<MODE_W, QK_SIGN>, a, grid, slots, s);
-    if (mode == MODE_W && a.q.kind == QK_UNIF) return grouped_launch(worker_grouped_kernel<MODE_W, QK_UNIF>, a, grid, slots, s);
-    if (mode == MODE_S && a.q.kind == QK_SIGN) return grouped_launch(worker_grouped_kernel<MODE_S, QK_SIGN>, a, grid, slots, s);
-    if (mode == MODE_S && a.q.kind == QK_UNIF) return grouped_launch(worker_grouped_kernel<MODE_S, QK_UNIF>, a, grid, slots, s);
-    return cudaErrorNotSupported;
+    if (a.q.kind != QK_UNIF) return cudaErrorNotSupported;
+    return mode == MODE_W ? grouped_launch(worker_grouped_kernel<MODE_W, QK_UNIF>, a, grid, slots, s)
+                          : grouped_launch(worker_grouped_kernel<MODE_S, QK_UNIF>, a, grid, slots, s);
 }
 
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s)

@@ -45,9 +45,12 @@ def test_ragged_sizes(d, group):
     _run_host(cfg, 3, seed=d)
 
 
-@pytest.mark.parametrize("n", [1, 2, 5, 8, 9, 16])
-def test_worker_counts(n):
-    cfg = ea.EAConfig(d=9000, n=n, qw=W.sign_q(4096), qs=W.sign_q(4096), alpha=1e-2)
+@pytest.mark.parametrize("n", [1, 2, 5, 8, 9, 16, 33])
+@pytest.mark.parametrize("group", [4096, 0])
+def test_worker_counts(n, group):
+    """Worker counts around the server's 8-worker sign table, with tile and whole-vector scales
+    (33 one-bit workers no longer fit the lazy broadcast's shared-memory staging)."""
+    cfg = ea.EAConfig(d=9000, n=n, qw=W.sign_q(group), qs=W.sign_q(group), alpha=1e-2)
     _run_host(cfg, 4, seed=n)
 
 
