@@ -85,6 +85,15 @@ __device__ __forceinline__ void cp_async4(void *dst, const void *src)
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
 }
 
+// 16-byte asynchronous copy global -> shared (both addresses 16-byte aligned; cached in L2 only).
+__device__ __forceinline__ void cp_async16(void *dst, const void *src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+
+// Wait until every cp.async this thread issued has landed in shared memory.
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 // One arrival on `bar` once every cp.async this thread issued before has landed (the barrier's
 // expected count already includes it).
 __device__ __forceinline__ void cp_async_arrive_noinc(uint64_t *bar)

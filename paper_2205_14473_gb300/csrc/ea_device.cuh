@@ -144,6 +144,28 @@ __device__ __forceinline__ float block_sign_scale(DF v, int64_t len, DF *red256,
     return *bcastf;
 }
 
+// CTA-wide compensated sum of the 256 threads' pairs, combined by warp 0 as in block_sign_scale
+// (eight pairs per lane in a tree, then five shuffle levels); the result is valid in thread 0
+// only.  One barrier; red256 may be reused after the next barrier.
+__device__ __forceinline__ DF block_sum_lane0(DF v, DF *red256)
+{
+    red256[threadIdx.x] = v;
+    compute_sync();
+    DF t{0.0f, 0.0f};
+    if (threadIdx.x < 32) {
+        DF p[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) p[j] = red256[threadIdx.x + 32 * j];
+        t = df_add(df_add(df_add(p[0], p[1]), df_add(p[2], p[3])), df_add(df_add(p[4], p[5]), df_add(p[6], p[7])));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            DF w{__shfl_down_sync(0xffffffffu, t.hi, o), __shfl_down_sync(0xffffffffu, t.lo, o)};
+            t = df_add(t, w);
+        }
+    }
+    return t;
+}
+
 // CTA-wide maximum for a group that is exactly this CTA's tile: one barrier, every thread combines
 // the warp maxima itself.  The caller must barrier before `red` is reused.
 __device__ __forceinline__ float block_max_all(float a, uint32_t *red)

@@ -401,17 +401,18 @@ __device__ __forceinline__ bool server_u_staged(const ServerArgs &a, int64_t til
         const int64_t cbase = tile * chunk_words;          // the tile's chunk in every code stream
         const int64_t avail = a.wcode_bytes / 4 - cbase;   // words of the (padded) stream from there
         const int nvec = n * chunk_words / 4;
+        // every copy issued at once (cp.async: no register round trip), then one wait
         for (int v = threadIdx.x; v < nvec; v += kThreads) {
             const int w = (4 * v) / chunk_words, o = (4 * v) % chunk_words;
-            uint4 c = make_uint4(0u, 0u, 0u, 0u);
-            if (o + 4 <= avail)
-                c = __ldg(reinterpret_cast<const uint4 *>(a.wwords + static_cast<int64_t>(w) * a.wwords_stride + cbase + o));
-            reinterpret_cast<uint4 *>(cw)[v] = c;
+            uint4 *dst = reinterpret_cast<uint4 *>(cw) + v;
+            if (o + 4 <= avail) cp_async16(dst, a.wwords + static_cast<int64_t>(w) * a.wwords_stride + cbase + o);
+            else *dst = make_uint4(0u, 0u, 0u, 0u);
         }
         if (has_scale<QW>())
             for (int i = threadIdx.x; i < n * ngw; i += kThreads)
-                wsc[i] = __ldg(a.wscales + static_cast<int64_t>(i / ngw) * a.wscales_stride + gw0 + i % ngw);
+                cp_async4(wsc + i, a.wscales + static_cast<int64_t>(i / ngw) * a.wscales_stride + gw0 + i % ngw);
         if (seg) cache_tile_groups(GW, tile, d, gs.tg);
+        cp_async_wait_all();
     }
     compute_sync();
     float acc[kSlots][4];

@@ -213,11 +213,12 @@ constexpr int PASS_LAZY_ONE = 16;
 // tile loop is instruction-bound).
 // PASS: PASS_FUSED or PASS_STASH as a compile-time constant (the other path is then not compiled
 // in), or -1 to follow `pass`.
+// part_idx (PASS_LAZY_ONE): where the tile's partial norm goes, looked up early by the caller.
 template <int QK, bool FULL = false, bool BALLOT = true, int PASS = -1, class USrc>
 __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64_t d, const QParams &q,
                                             uint32_t *words, float *scales, float *resid, int ef, int pass,
                                             uint64_t seed, uint32_t id, uint32_t t, double *partials,
-                                            TileSmem &sm)
+                                            TileSmem &sm, int64_t part_idx = 0)
 {
     if constexpr (PASS >= 0) pass = PASS;
     if constexpr (!has_scale<QK>()) {
@@ -256,8 +257,8 @@ __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64
             return;
         }
         if constexpr (PASS == PASS_LAZY_ONE && QK == QK_SIGN) {
-            // u (with error feedback), the codes, and the one group's partial norm of the tile --
-            // the same sum, in the same order, as the per-group loop below forms
+            // u (with error feedback), the codes, and the one group's partial norm of the tile
+            // (a compensated sum to ~2^-44, like the per-group loop below; one barrier)
             DF acc{0.0f, 0.0f};
 #pragma unroll
             for (int k = 0; k < kSlots; ++k) {
@@ -275,12 +276,8 @@ __device__ __forceinline__ void finish_tile(const USrc &src, int64_t tile, int64
                 }
                 store_codes4<FULL, BALLOT>(words, qs, 1, c, 0, d);
             }
-            const double part = block_sum(acc, sm.red, &sm.bcast);
-            if (threadIdx.x == 0) {
-                const Grouping &G = q.grp;
-                const int64_t g = first_group_of_tile(G, tile);
-                partials[G.pair_base[g] + (tile - group_begin(G, g, d) / kTile)] = part;
-            }
+            const DF tot = block_sum_lane0(acc, sm.red256);
+            if (threadIdx.x == 0) partials[part_idx] = static_cast<double>(tot.hi) + static_cast<double>(tot.lo);
             return;
         }
         // PASS_STASH: u into resid for encode_kernel.  PASS_LAZY (scaled sign): u into resid, where
@@ -375,27 +372,29 @@ __device__ __forceinline__ void lazy_residual4(const QParams &q, const float *sc
 }
 
 // The same for all of this thread's slots of tile `tile`.
-// ONE: the tile lies inside one group (no per-coordinate lookups are compiled in).
-template <bool FULL, bool ONE = false>
+// The same for a tile inside one group, whose previous scale is s.
+template <bool FULL>
+__device__ __forceinline__ void lazy_residual_one(const QParams &q, float s, int64_t tile, int64_t d,
+                                                  float (&e)[kSlots][4])
+{
+#pragma unroll
+    for (int k = 0; k < kSlots; ++k) {
+        const int64_t j0 = 4 * slot_of(tile, k);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (FULL || j0 + i < d) {
+                float dec;
+                (void)encode1<QK_SIGN>(e[k][i], s, q, 0.0f, 0, 0.0f, dec);
+                e[k][i] = __fsub_rn(e[k][i], dec);
+            }
+        }
+    }
+}
+
+template <bool FULL>
 __device__ __forceinline__ void lazy_residual(const QParams &q, const float *scales, int64_t tile, int64_t d,
                                               float (&e)[kSlots][4])
 {
-    if constexpr (ONE) {
-        const float s = scales[first_group_of_tile(q.grp, tile)];
-#pragma unroll
-        for (int k = 0; k < kSlots; ++k) {
-            const int64_t j0 = 4 * slot_of(tile, k);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                if (FULL || j0 + i < d) {
-                    float dec;
-                    (void)encode1<QK_SIGN>(e[k][i], s, q, 0.0f, 0, 0.0f, dec);
-                    e[k][i] = __fsub_rn(e[k][i], dec);
-                }
-            }
-        }
-        return;
-    }
     const LazyScale ls = lazy_scale_of_tile(q, scales, tile, d);
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) lazy_residual4<FULL>(q, scales, ls, 4 * slot_of(tile, k), d, e[k]);

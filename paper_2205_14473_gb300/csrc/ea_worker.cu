@@ -10,6 +10,16 @@ template <int MODE, int QK, bool FULL, int PASS>
 __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, float4 *ubuf, TileSmem &sm)
 {
     const int64_t d = a.d;
+    // PASS_LAZY_ONE: the tile's group, its previous scale and the slot of its partial norm, looked
+    // up before the tile's loads so that these short dependent loads overlap them
+    int64_t part_idx = 0;
+    float s_prev = 0.0f;
+    if constexpr (PASS == PASS_LAZY_ONE) {
+        const Grouping &G = a.q.grp;
+        const int64_t g1 = first_group_of_tile(G, tile);
+        part_idx = G.pair_base[g1] + (tile - group_begin(G, g1, d) / kTile);
+        if (a.lazy_in) s_prev = a.scales[g1];
+    }
     float g[kSlots][4], e[kSlots][4], m[kSlots][4], v[kSlots][4];
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
@@ -24,9 +34,11 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
     // the grid's fl(i/L) table, built while the loads are in flight (read after the scale
     // reduction's barrier)
     build_qtab<QK>(a.q, sm.qtab);
-    if constexpr (PASS == PASS_LAZY || PASS == PASS_LAZY_ONE) {
+    if constexpr (PASS == PASS_LAZY) {
         // e holds the previous round's u: its residual is u - Q(u) with the previous scales
-        if (a.lazy_in) lazy_residual<FULL, PASS == PASS_LAZY_ONE>(a.q, a.scales, tile, d, e);
+        if (a.lazy_in) lazy_residual<FULL>(a.q, a.scales, tile, d, e);
+    } else if constexpr (PASS == PASS_LAZY_ONE) {
+        if (a.lazy_in) lazy_residual_one<FULL>(a.q, s_prev, tile, d, e);
     }
 #pragma unroll
     for (int k = 0; k < kSlots; ++k) {
@@ -46,7 +58,7 @@ __device__ __forceinline__ void worker_tile(const WorkerArgs &a, int64_t tile, f
         }
     }
     finish_tile<QK, FULL, true, PASS>(USmem{ubuf}, tile, d, a.q, a.words, a.scales, a.e, a.ef, a.pass, a.seed, a.id, a.t,
-                          a.partials, sm);
+                                      a.partials, sm, part_idx);
 }
 
 // Algorithm 2 for one worker on one 4096-coordinate tile.  With Adam at the worker:
