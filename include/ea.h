@@ -130,9 +130,10 @@ int ea_round_index(const ea_handle *h, int64_t *t);
 /* Kernel launches that one round makes on the stream: n worker compresses, one server step and one
  * apply.  A message whose scale groups lie inside 4096-coordinate tiles takes one launch.  When the
  * groups span tiles:
- *   - a scaled-sign message takes two: one pass writes the codes (the signs, which need no scale)
- *     with the groups' partial norms, and a finalize forms the scales (the residual is formed from
- *     the kept input where it is next read; see the residual views);
+ *   - a scaled-sign message takes one pass, which writes the codes (the signs, which need no scale)
+ *     with the groups' partial norms, and a finalize forms the scales: one finalize for all worker
+ *     messages (at the server step, or at a view of a worker's scales or residual), one for the
+ *     broadcast (the residual is formed from the kept input where it is next read; see the views);
  *   - another message takes one launch in the grouped kernel, which holds u in shared memory while
  *     the partial norms are combined, when its waves fit: for the broadcast, groups of up to ~7.5
  *     million coordinates on a GB300; for a worker message, no more 4096-tiles than the grouped

@@ -59,7 +59,8 @@ struct ea_handle {
     float *m = nullptr, *v = nullptr, *e = nullptr, *es = nullptr, *ms = nullptr, *vs = nullptr;
     uint32_t *wcodes = nullptr, *scodes = nullptr;
     float *wscales = nullptr, *sscales = nullptr;
-    double *partials = nullptr;
+    double *partials = nullptr;   // the worker messages' partial norms (one set each when lazy)
+    double *spartials = nullptr;  // the broadcast's
     uint32_t *status = nullptr;
     float *rview = nullptr;  // PASS_LAZY: the residual views are formed here
     StagePlan splan{};
@@ -70,6 +71,7 @@ struct ea_handle {
     std::vector<unsigned char> lazy_w;  // PASS_LAZY: worker i's e holds its last u (see lazy_residual)
     bool lazy_s = false;                // PASS_LAZY: e_s holds the last w
     bool lazy_staged = false;           // PASS_LAZY broadcast: every tile's worker messages fit the staging
+    bool wscales_pending = false;       // PASS_LAZY workers: a message's scales are not formed yet
     int n_compressed = 0;
     bool has_message = false;
     uint64_t up_bits = 0, down_bits = 0;
@@ -238,7 +240,12 @@ Layout make_layout(const ea_config &c, const QHost &qw, const QHost &qs)
     L.scales_w = static_cast<size_t>(L.wscale_stride) * 4 * c.n;
     L.codes_s = align_up(static_cast<size_t>(qs.n_words) * 4, kAlign);
     L.scales_s = align_up(static_cast<size_t>(std::max<int64_t>(qs.n_groups, 1)) * 4, kAlign);
-    L.partials = static_cast<size_t>(std::max(qw.n_pairs, qs.n_pairs)) * sizeof(double);
+    // partial norms: shared by the messages one after another, except that lazy scaled-sign worker
+    // messages keep one set each (their scales are formed together before the server step) and the
+    // broadcast then has its own
+    const bool lazy_w = qw.pass == PASS_STASH && qw.kind == EA_Q_SIGN_L1;
+    L.partials = (lazy_w ? static_cast<size_t>(c.n) * qw.n_pairs + qs.n_pairs
+                         : static_cast<size_t>(std::max(qw.n_pairs, qs.n_pairs))) * sizeof(double);
     L.off_w = qw.gkind == GK_SEG ? qw.offsets.size() * 8 : 0;
     L.tg_w = qw.gkind == GK_SEG ? static_cast<size_t>(n_tiles) * 4 : 0;
     L.pb_w = qw.pass == PASS_STASH ? qw.pair_base.size() * 8 : 0;
@@ -465,19 +472,38 @@ int check_dev_ptr(ea_handle *h, const void *p, const char *what)
 
 // Finish a message whose scale groups span tiles: scales from the partial norms, then encode.
 // The group scales from the per-(tile, group) partial norms (PASS_STASH, PASS_LAZY).
-int finalize_scales(ea_handle *h, const QHost &q, float *scales)
+int finalize_scales(ea_handle *h, const QHost &q, const double *partials, float *scales)
 {
     FinalizeArgs f{};
     f.d = h->cfg.d;
     f.q = device_quant(q);
-    f.partials = h->partials;
+    f.partials = partials;
     f.scales = scales;
     return check_cuda(h, launch_finalize(f, h->stream), "finalize launch");
 }
 
-int second_pass(ea_handle *h, const QHost &q, float *buf, uint32_t *words, float *scales, uint32_t id)
+// PASS_LAZY worker messages: the scales of all n messages in one launch, from each worker's own
+// partial norms (a message compressed in an earlier round gets the same scales again).
+int finalize_worker_scales(ea_handle *h)
 {
-    int r = finalize_scales(h, q, scales);
+    if (!h->wscales_pending) return EA_OK;
+    FinalizeArgs f{};
+    f.d = h->cfg.d;
+    f.q = device_quant(h->qw);
+    f.partials = h->partials;
+    f.scales = h->wscales;
+    f.n_msgs = h->cfg.n;
+    f.partials_stride = h->qw.n_pairs;
+    f.scales_stride = h->lay.wscale_stride;
+    const int r = check_cuda(h, launch_finalize(f, h->stream), "finalize launch");
+    if (r == EA_OK) h->wscales_pending = false;
+    return r;
+}
+
+int second_pass(ea_handle *h, const QHost &q, const double *partials, float *buf, uint32_t *words, float *scales,
+                uint32_t id)
+{
+    int r = finalize_scales(h, q, partials, scales);
     if (r != EA_OK) return r;
     EncodeArgs e{};
     e.d = h->cfg.d;
@@ -594,6 +620,7 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->scodes = reinterpret_cast<uint32_t *>(take(L.codes_s));
     h->sscales = reinterpret_cast<float *>(take(L.scales_s));
     h->partials = reinterpret_cast<double *>(take(L.partials));
+    h->spartials = h->partials;
     h->qw.d_offsets = reinterpret_cast<int64_t *>(take(L.off_w));
     h->qw.d_tile_group = reinterpret_cast<int32_t *>(take(L.tg_w));
     h->qw.d_pair_base = reinterpret_cast<int64_t *>(take(L.pb_w));
@@ -608,7 +635,10 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
     h->rview = reinterpret_cast<float *>(take(L.rview));
     // scaled-sign messages whose groups span tiles: the sign codes need no scale, so one pass writes
     // them and keeps u (PASS_LAZY); its workspace is that of the two passes
-    if (h->qw.pass == PASS_STASH && h->qw.kind == EA_Q_SIGN_L1) h->qw.pass = PASS_LAZY;
+    if (h->qw.pass == PASS_STASH && h->qw.kind == EA_Q_SIGN_L1) {
+        h->qw.pass = PASS_LAZY;
+        h->spartials = h->partials + static_cast<int64_t>(cfg->n) * h->qw.n_pairs;
+    }
     if (h->qs.pass == PASS_STASH && h->qs.kind == EA_Q_SIGN_L1) {
         h->qs.pass = PASS_LAZY;
         // the server stages a tile's worker codes and scales in shared memory when they fit
@@ -687,7 +717,7 @@ int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
     a.seed = h->cfg.seed;
     a.id = static_cast<uint32_t>(worker);
     a.t = static_cast<uint32_t>(h->t);
-    a.partials = h->partials;
+    a.partials = h->qw.pass == PASS_LAZY ? h->partials + static_cast<int64_t>(worker) * h->qw.n_pairs : h->partials;
     a.status = h->status;
     a.lazy_in = h->qw.pass == PASS_LAZY ? h->lazy_w[worker] : 0;
     if (h->qw.pass == PASS_GROUPED) {
@@ -697,10 +727,12 @@ int ea_worker_compress(ea_handle *h, int32_t worker, const float *g)
     } else {
         r = check_cuda(h, launch_worker(W ? MODE_W : MODE_S, a, h->stream), "worker launch");
     }
-    if (r == EA_OK && h->qw.pass == PASS_STASH) r = second_pass(h, h->qw, a.e, a.words, a.scales, a.id);
-    if (r == EA_OK && h->qw.pass == PASS_LAZY) r = finalize_scales(h, h->qw, a.scales);
+    if (r == EA_OK && h->qw.pass == PASS_STASH) r = second_pass(h, h->qw, a.partials, a.e, a.words, a.scales, a.id);
     if (r != EA_OK) return r;
-    if (h->qw.pass == PASS_LAZY) h->lazy_w[worker] = h->cfg.error_feedback ? 1 : 0;
+    if (h->qw.pass == PASS_LAZY) {  // the scales are formed for all workers before the server step
+        h->lazy_w[worker] = h->cfg.error_feedback ? 1 : 0;
+        h->wscales_pending = true;
+    }
     h->compressed[worker] = 1;
     ++h->n_compressed;
     return EA_OK;
@@ -732,19 +764,20 @@ int ea_server_step(ea_handle *h)
     a.pass = h->qs.pass;
     a.seed = h->cfg.seed;
     a.t = static_cast<uint32_t>(h->t);
-    a.partials = h->partials;
+    a.partials = h->spartials;
     a.dpad = h->lay.dpad;
     a.wcode_bytes = h->lay.wcode_stride * 4;
     a.status = h->status;
     a.plan = h->splan;
     a.lazy_in = h->qs.pass == PASS_LAZY && h->lazy_s ? 1 : 0;
     const bool W = h->cfg.placement == EA_ADAM_AT_WORKER;
-    int r;
+    int r = finalize_worker_scales(h);
+    if (r != EA_OK) return r;
     if (h->qs.pass == PASS_LAZY) {
         r = check_cuda(h, W ? launch_server_lazy<MODE_W>(a, h->lazy_staged, h->stream)
                             : launch_server_lazy<MODE_S>(a, h->lazy_staged, h->stream),
                        "server launch");
-        if (r == EA_OK) r = finalize_scales(h, h->qs, h->sscales);
+        if (r == EA_OK) r = finalize_scales(h, h->qs, h->spartials, h->sscales);
         if (r == EA_OK) h->lazy_s = h->cfg.error_feedback != 0;
     } else if (h->qs.pass == PASS_GROUPED) {
         a.gp = device_group_plan(h->qs, h->epoch_s);
@@ -754,7 +787,7 @@ int ea_server_step(ea_handle *h)
         r = check_cuda(h, launch_server(W ? MODE_W : MODE_S, a, h->stream), "server launch");
     }
     if (r == EA_OK && h->qs.pass == PASS_STASH)
-        r = second_pass(h, h->qs, h->es, h->scodes, h->sscales, static_cast<uint32_t>(h->cfg.n));
+        r = second_pass(h, h->qs, h->spartials, h->es, h->scodes, h->sscales, static_cast<uint32_t>(h->cfg.n));
     if (r != EA_OK) return r;
     h->up_bits += static_cast<uint64_t>(h->cfg.n) * message_bits(h->qw, h->cfg.d);
     h->down_bits += static_cast<uint64_t>(h->cfg.n) * message_bits(h->qs, h->cfg.d);
@@ -808,7 +841,9 @@ int ea_round_launches(const ea_handle *h, int32_t *launches)
 {
     if (!h || !launches) return fail(nullptr, EA_E_INVAL, "NULL argument");
     auto per_message = [](const QHost &q) { return q.pass == PASS_STASH ? 3 : q.pass == PASS_LAZY ? 2 : 1; };
-    *launches = h->cfg.n * per_message(h->qw) + per_message(h->qs) + 1;
+    // lazy worker messages: one pass each, and one finalize for all of them
+    const int workers = h->qw.pass == PASS_LAZY ? h->cfg.n + 1 : h->cfg.n * per_message(h->qw);
+    *launches = workers + per_message(h->qs) + 1;
     return EA_OK;
 }
 
@@ -830,6 +865,12 @@ int ea_get_view(const ea_handle *h, int32_t which, int32_t index, void **dev_ptr
         return fail(hm, EA_E_INVAL, "worker %d out of [0, %d)", index, h->cfg.n);
     const int64_t dp = h->lay.dpad;
     const size_t vec = static_cast<size_t>(h->cfg.d) * 4;
+    if ((which == EA_VIEW_SCALES_WORKER || which == EA_VIEW_E_WORKER) && h->wscales_pending) {
+        // lazy worker messages compressed this round: their scales first
+        int r = finalize_worker_scales(hm);
+        if (r == EA_OK) r = check_cuda(hm, cudaStreamSynchronize(h->stream), "stream synchronize");
+        if (r != EA_OK) return r;
+    }
     void *p = nullptr;
     size_t n = 0;
     switch (which) {

@@ -175,11 +175,15 @@ struct EncodeArgs {
     uint32_t id, t;
 };
 
+// The scales of n_msgs messages (blockIdx.y; 0 counts as 1), message y's partials at
+// partials + y * partials_stride and its scales at scales + y * scales_stride.
 struct FinalizeArgs {
     int64_t d;
     QParams q;
     const double *partials;
     float *scales;
+    int n_msgs;
+    int64_t partials_stride, scales_stride;
 };
 
 // PASS_LAZY: the residual u - Q(u) of the u kept in `u`, with the scales of its message, into out.

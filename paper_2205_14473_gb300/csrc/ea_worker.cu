@@ -187,8 +187,9 @@ __global__ void __launch_bounds__(kThreads, MODE == MODE_S ? 4 : 2) worker_group
     }
 }
 
-// Second pass, one CTA per scale group: combine the group's per-tile partial norms in a fixed
-// order and write the group scale (Example 1: ||.||_inf; scaled sign: ||.||_1 / |group|).
+// One CTA per scale group (blockIdx.x) and message (blockIdx.y): combine the group's per-tile
+// partial norms in a fixed order and write the group scale (Example 1: ||.||_inf; scaled sign:
+// ||.||_1 / |group|).
 template <int QK>
 __global__ void __launch_bounds__(kThreads) finalize_kernel(const FinalizeArgs a)
 {
@@ -196,10 +197,12 @@ __global__ void __launch_bounds__(kThreads) finalize_kernel(const FinalizeArgs a
     pdl_trigger();
     pdl_wait();
     const int64_t gi = blockIdx.x;
+    const double *partials = a.partials + static_cast<int64_t>(blockIdx.y) * a.partials_stride;
+    float *scales = a.scales + static_cast<int64_t>(blockIdx.y) * a.scales_stride;
     const int64_t pb = a.q.grp.pair_base[gi], pe = a.q.grp.pair_base[gi + 1];
     double acc = 0.0;
     for (int64_t p = pb + threadIdx.x; p < pe; p += kThreads)
-        acc = (QK == QK_SIGN) ? __dadd_rn(acc, a.partials[p]) : fmax(acc, a.partials[p]);
+        acc = (QK == QK_SIGN) ? __dadd_rn(acc, partials[p]) : fmax(acc, partials[p]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const double w = __shfl_down_sync(0xffffffffu, acc, o);
@@ -211,7 +214,7 @@ __global__ void __launch_bounds__(kThreads) finalize_kernel(const FinalizeArgs a
         double t = red[0];
         for (int w = 1; w < kWarps; ++w) t = (QK == QK_SIGN) ? __dadd_rn(t, red[w]) : fmax(t, red[w]);
         const int64_t len = group_end(a.q.grp, gi, a.d) - group_begin(a.q.grp, gi, a.d);
-        a.scales[gi] = (QK == QK_SIGN) ? sign_scale(t, len) : static_cast<float>(t);
+        scales[gi] = (QK == QK_SIGN) ? sign_scale(t, len) : static_cast<float>(t);
     }
 }
 
@@ -425,7 +428,8 @@ cudaError_t launch_worker_grouped(int mode, const WorkerArgs &a, int grid, cudaS
 
 cudaError_t launch_finalize(const FinalizeArgs &a, cudaStream_t s)
 {
-    const dim3 grid(static_cast<unsigned>(a.q.grp.n_groups)), block(kThreads);
+    const dim3 grid(static_cast<unsigned>(a.q.grp.n_groups), static_cast<unsigned>(a.n_msgs > 1 ? a.n_msgs : 1)),
+        block(kThreads);
     if (a.q.kind == QK_SIGN) return launch_pdl(finalize_kernel<QK_SIGN>, grid, block, 0, s, a);
     return launch_pdl(finalize_kernel<QK_UNIF>, grid, block, 0, s, a);
 }

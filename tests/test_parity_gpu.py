@@ -138,32 +138,34 @@ def test_two_pass_scale_beyond_the_grouped_capacity():
     """A whole-vector scale over 12.3 million coordinates: more tiles than the one-pass grouped
     kernels hold in shared memory at once (about 1,800 on a GB300).  The uniform-grid broadcast
     takes the two-pass scale (stash, finalize, encode: three launches); the scaled-sign worker
-    messages take the lazy pass (codes with the partial norms, then finalize: two launches)."""
+    messages take the lazy pass (codes with the partial norms: one launch each, and one finalize
+    for all of them)."""
     d = 3000 * 4096 + 3
     cfg = ea.EAConfig(d=d, n=2, qw=W.sign_q(0), qs=W.uniform_q(8, 0, False), alpha=1e-3, seed=41)
     L = _run_host(cfg, 3, seed=43)
-    assert L.gpu.launches_per_round == 2 * 2 + 3 + 1
+    assert L.gpu.launches_per_round == 2 + 1 + 3 + 1
 
 
-@pytest.mark.parametrize("qw,qs,launches", [(W.sign_q(0), W.sign_q(0), 3 * 2 + 2 + 1),
+@pytest.mark.parametrize("qw,qs,launches", [(W.sign_q(0), W.sign_q(0), 3 + 1 + 2 + 1),
                                            (W.uniform_q(4, 0, True), W.uniform_q(8, 1000, False), 3 * 1 + 1 + 1)])
 def test_grouped_scales_one_launch_per_message(qw, qs, launches):
     """Scale groups that span tiles (74 tiles): uniform-grid messages take the one-pass grouped
     kernels (one tile per worker CTA, one launch each); scaled-sign messages take the lazy pass (the
-    signs with the partial norms, then finalize: two launches each)."""
+    signs with the partial norms; one finalize forms the scales of all worker messages, another
+    the broadcast's)."""
     cfg = ea.EAConfig(d=300_001, n=3, qw=qw, qs=qs, alpha=1e-3, seed=45)
     L = _run_host(cfg, 3, seed=47)
     assert L.gpu.launches_per_round == launches
 
 
 @pytest.mark.parametrize("qw,qs,placement,launches", [
-    (W.sign_q(0), W.sign_q(0), ea.ADAM_AT_WORKER, 3 * 2 + 2 + 1),
+    (W.sign_q(0), W.sign_q(0), ea.ADAM_AT_WORKER, 3 + 1 + 2 + 1),
     (W.uniform_q(4, 0, True), W.uniform_q(8, 0, False), ea.ADAM_AT_SERVER, 3 * 3 + 1 + 1),
     (W.uniform_q(4, 0, True), W.uniform_q(8, 0, False), ea.ADAM_AT_WORKER, 3 * 3 + 1 + 1),
     (W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)), W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)),
-     ea.ADAM_AT_WORKER, 3 * 2 + 2 + 1),
+     ea.ADAM_AT_WORKER, 3 + 1 + 2 + 1),
     (W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)), W.sign_q(-1, (1_500_007, 64, 2_000_000, 128, 900_001)),
-     ea.ADAM_AT_SERVER, 3 * 2 + 2 + 1),
+     ea.ADAM_AT_SERVER, 3 + 1 + 2 + 1),
 ])
 def test_grouped_broadcast_with_several_tiles_per_cta(qw, qs, placement, launches):
     """4.4 million coordinates (1,075 tiles).  A uniform-grid broadcast takes the grouped kernel,
@@ -174,6 +176,40 @@ def test_grouped_broadcast_with_several_tiles_per_cta(qw, qs, placement, launche
     cfg = ea.EAConfig(d=d, n=3, qw=qw, qs=qs, alpha=1e-3, placement=placement, seed=49)
     L = _run_host(cfg, 3, seed=51)
     assert L.gpu.launches_per_round == launches
+
+
+@pytest.mark.parametrize("group", [0, -1])
+def test_lazy_views_mid_round_change_nothing(group):
+    """Lazy scaled-sign messages: viewing a worker's scales and residual between its compress and the
+    server step forms them early (the view matches the values after the round), and the state of a
+    handle viewed that way stays bit-identical to that of one never viewed."""
+    d = 50_003
+    segs = (20_000, 64, 29_939) if group < 0 else ()
+    q = W.sign_q(group, segs) if group < 0 else W.sign_q(0)
+    cfg = ea.EAConfig(d=d, n=3, qw=q, qs=q, alpha=1e-3, seed=5)
+    a, b = ea.EARound(cfg), ea.EARound(cfg)
+    gen = torch.Generator(device="cuda").manual_seed(7)
+    xa, xb = torch.zeros(d, device="cuda"), torch.zeros(d, device="cuda")
+    for t in range(4):
+        g = [torch.randn(d, device="cuda", generator=gen) for _ in range(cfg.n)]
+        for i in range(cfg.n):
+            a.worker_compress(i, g[i])
+            b.worker_compress(i, g[i])
+        mid = [(a.view(ea.EA_VIEW_SCALES_WORKER, i).clone(), a.view(ea.EA_VIEW_E_WORKER, i)[:d].clone())
+               for i in range(cfg.n)]
+        for r, x in ((a, xa), (b, xb)):
+            r.server_step()
+            r.apply(x)
+        torch.cuda.synchronize()
+        for i in range(cfg.n):
+            assert torch.equal(a.view(ea.EA_VIEW_SCALES_WORKER, i), mid[i][0])
+            assert torch.equal(a.view(ea.EA_VIEW_E_WORKER, i)[:d], mid[i][1])
+            for v in (ea.EA_VIEW_CODES_WORKER, ea.EA_VIEW_SCALES_WORKER, ea.EA_VIEW_E_WORKER):
+                assert torch.equal(a.view(v, i), b.view(v, i))
+        for v in (ea.EA_VIEW_CODES_SERVER, ea.EA_VIEW_SCALES_SERVER, ea.EA_VIEW_E_SERVER):
+            assert torch.equal(a.view(v), b.view(v))
+        assert torch.equal(xa, xb)
+    assert a.launches_per_round == cfg.n + 1 + 2 + 1
 
 
 def test_replicas_are_identical_and_protocol():
@@ -226,7 +262,7 @@ def test_c1_full():
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
     assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (2_622_720, 2_622_720)
-    assert L.gpu.launches_per_round == 2 * w.n + 2 + 1  # scaled-sign messages: the lazy pass + finalize
+    assert L.gpu.launches_per_round == w.n + 1 + 2 + 1  # scaled-sign messages: the lazy pass + finalize
 
 
 def test_c2_quadratic_toy_full():
@@ -267,8 +303,9 @@ def test_c3_resnet18_all_tensors(placement, rounds):
         _dev_grads(w, t, bufs)
         L.round(bufs, [L.host(b) for b in bufs], x_dev, x_host)
     assert L.total_mismatch == 0
-    # per-tensor scales: every message in the lazy pass (codes and partial norms, then finalize)
-    assert L.gpu.launches_per_round == 2 * w.n + 2 + 1
+    # per-tensor scales: every message in the lazy pass (codes and partial norms), one finalize for
+    # the worker messages' scales and one for the broadcast's
+    assert L.gpu.launches_per_round == w.n + 1 + 2 + 1
     if rounds == w.rounds:
         assert L.gpu.bits_sent() == expected_bits(cfg, w.rounds) == (18_706_393_600, 18_706_393_600)
 
