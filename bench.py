@@ -115,9 +115,9 @@ def _ncu_traffic(kernel: str, workload: str, placement: int):
     return None
 
 
-# The kernels behind each step of a round (a message of the two-pass scale is three launches).
-ROLE_KERNELS = {"compress": ("worker_kernel", "worker_grouped", "finalize_kernel", "encode_kernel"),
-                "server": ("server_staged", "server_grouped", "server_kernel"),
+# The kernels behind each step of a round (the finalize launches, which move a few KB, are left out).
+ROLE_KERNELS = {"compress": ("worker_kernel", "worker_grouped", "worker_lazy", "encode_kernel"),
+                "server": ("server_staged", "server_grouped", "server_lazy", "server_kernel"),
                 "apply": ("apply_kernel",)}
 
 
