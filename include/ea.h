@@ -100,7 +100,9 @@ int ea_init(const ea_config *cfg, void *workspace, size_t workspace_bytes, void 
  * keep e <- u - Q_w(u).  g: d binary32 values, 16-byte aligned, read only, not retained; device
  * memory, or pinned host memory mapped into the device's address space (the kernel then reads it
  * over the host link, with no staging copy).  Each worker compresses once per round; EA_E_ORDER
- * otherwise. */
+ * otherwise.  A scaled-sign message whose scale groups span 4096-coordinate tiles has its codes when
+ * this returns; its scales are formed, with those of the other workers' messages, by the next
+ * ea_server_step (or by a view of them, see ea_get_view), and e is kept as u (see ea_get_view). */
 int ea_worker_compress(ea_handle *h, int32_t worker, const float *g);
 
 /* Algorithm 1: average the n decoded worker messages (summed in worker order, then divided by
