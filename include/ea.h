@@ -173,7 +173,8 @@ int ea_sync_status(ea_handle *h);
 #define EA_NOALLOC_MAX_D ((int64_t)16384 * 4096)
 
 /* The paper has no counterpart: this is a deployment convenience.  Worker compress (the same
- * computation as ea_worker_compress, with the same kernels) for callers that cannot allocate
+ * computation as ea_worker_compress, with the same results; it always takes the two-pass scale --
+ * stash, finalize, encode -- and leaves the residual e itself in its buffer) for callers that cannot allocate
  * device memory -- code running inside a framework whose caching allocator has already reserved
  * the GPU's memory, latency-critical paths that must not take cudaMalloc's implicit
  * synchronisation, or plug-ins that are handed only the buffers they work on.  It needs no handle

@@ -10,7 +10,9 @@
 // into the library: every GPU that loads the library holds it (128 KB + 256 B) until the process
 // exits, whether or not the function is called.
 //
-// The kernels are the ones ea_worker_compress launches; only where their scratch lives differs.
+// The kernels are those of the two-pass scale that ea_worker_compress also launches (for the
+// uniform grid; a scaled-sign message there takes the lazy pass, with the same results); only where
+// their scratch lives differs.
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
